@@ -1,0 +1,419 @@
+"""Benchmark of the AoH attention path on GB300.
+
+One "step" is one decode step of the Llama-3-8B-shaped decode workload
+(32 query / 8 KV heads, d_head 128, batch 16, every sequence at 128K cached
+tokens, 4 of 8 KV heads streaming with S=128, W=4096): the headline is
+decode attention us/step and its HBM GB/s. The same run times the
+Qwen2.5-7B-shaped 32K prefill (28 / 4 heads, 2 streaming, S=128, W=2048) for
+prefill attention TFLOP/s, reported in the "prefill" object.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
+
+--impl reference times the CPU float64 oracle on a bounded sample of the
+same decode step (no GPU needed). Multi-GPU runs (torchrun) are independent
+replicas of the per-GPU workload (weak scaling, no collective on the data
+path); rank 0 prints one JSON line.
+"""
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode attn µs/step & HBM GB/s @128K ctx; prefill attn TFLOP/s @32K"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "of measured"
+    return dict(FALLBACK_PEAKS), "of fallback"
+
+
+# ------------------------------------------------------------------ workload
+
+def decode_workload():
+    from paper_2608_06849_gb300.workloads import DECODE_128K, labels_for
+    wl = DECODE_128K
+    return wl, labels_for(wl)
+
+
+def prefill_workload():
+    from paper_2608_06849_gb300.workloads import PREFILL_32K, labels_for
+    wl = PREFILL_32K
+    return wl, labels_for(wl)
+
+
+def decode_bytes(lens_before, labels, wl):
+    """Algorithmic HBM bytes of one decode step: cached K/V rows read once,
+    the new token's K/V read and appended, q read, output written."""
+    D, g = wl.d_head, wl.g
+    row = D * 2
+    total = 0
+    for t in lens_before:
+        for lab in labels:
+            rows = (t + 1) if lab == 0 else min(t + 1, wl.sink + wl.window)
+            total += (rows - 1) * row * 2          # cached K and V rows
+            total += row * 2 * 2                   # new K/V read + appended
+        total += wl.n_q_heads * D * 2 * 2          # q read + out written
+    return total
+
+
+def attended_pairs(T, S, W, streaming):
+    """Number of (query, key) pairs a head attends in a causal prefill of T tokens."""
+    if not streaming:
+        return T * (T + 1) // 2
+    i = list(range(T))
+    tot = 0
+    for x in i:
+        sinks = min(x + 1, S)
+        lo = max(S, x - W + 1)
+        tot += sinks + max(0, x - lo + 1)
+    return tot
+
+
+def prefill_flops(wl, labels, T):
+    g = wl.g
+    pairs = sum(attended_pairs(T, wl.sink, wl.window, lab == 1) for lab in labels) * g
+    return 4.0 * wl.d_head * pairs
+
+
+# ------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.out = os.path.join("/tmp", f"aoh_clocks_{os.getpid()}.csv")
+        try:
+            self.f = open(self.out, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100", "-i", str(device_index)], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.out):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.out)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# -------------------------------------------------------------- native arm
+
+def run_native(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_06849_gb300 import aoh
+    from paper_2608_06849_gb300 import build as aoh_build
+    from paper_2608_06849_gb300.workloads import decode_inputs, randn_bf16
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    aoh_build.build()
+    aoh.load()
+    peaks, peak_note = load_peaks()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    stream = torch.cuda.current_stream()
+    K, W = args.steps, args.warmup
+
+    # ---------------- decode leg (headline)
+    wl, labels = decode_workload()
+    B, D, T0 = wl.batch, wl.d_head, wl.prefill_len
+    total_steps = W + K + K + 2   # warmup, timed, e2e
+    cache = aoh.Cache(B, wl.n_q_heads, wl.n_kv_heads, D, T0 + total_steps + 8, wl.sink, wl.window, labels)
+    kfill = randn_bf16((B, T0, wl.n_kv_heads, D), 7001 + rank, "cuda")
+    vfill = randn_bf16((B, T0, wl.n_kv_heads, D), 7002 + rank, "cuda")
+    cache.prefill(None, kfill, vfill, None)
+    torch.cuda.synchronize()
+    del kfill, vfill
+    torch.cuda.empty_cache()
+    inputs = [decode_inputs(wl, s, device="cuda") for s in range(W + K)]
+    out = torch.empty(B, wl.n_q_heads, D, dtype=torch.bfloat16, device="cuda")
+    for s in range(W):
+        cache.decode_step(*inputs[s], out)
+    cache.check()
+    lens_before = cache.lens()
+    step_bytes = []
+    for s in range(K):
+        step_bytes.append(decode_bytes([x + s for x in lens_before], labels, wl))
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    clocks = ClockSampler(local) if rank == 0 else None
+    barrier()
+    ev[0].record(stream)
+    for s in range(K):
+        cache.decode_step(*inputs[W + s], out)
+        ev[s + 1].record(stream)
+    barrier()
+    per_step_ms = [ev[s].elapsed_time(ev[s + 1]) for s in range(K)]
+    dec_ms = max_over_ranks(sum(per_step_ms))
+    cache.check()
+    dec_us_step = dec_ms * 1000.0 / K
+    avg_bytes = sum(step_bytes) / K
+    dec_gbs = avg_bytes / (dec_us_step * 1e-6) / 1e9
+
+    # e2e: same decode step through the C ABI from pinned host buffers
+    hq = [t.cpu().pin_memory() for t in inputs[W]]
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    dq = [torch.empty_like(t) for t in inputs[W]]
+    h2d = sum(t.numel() * t.element_size() for t in hq)
+    d2h = hout.numel() * hout.element_size()
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(K):
+        for dst, src in zip(dq, hq):
+            dst.copy_(src, non_blocking=True)
+        cache.decode_step(dq[0], dq[1], dq[2], out)
+        hout.copy_(out, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_us = max_over_ranks(e0.elapsed_time(e1)) * 1000.0 / K
+    cache.close()
+    del cache, inputs
+    torch.cuda.empty_cache()
+
+    # ---------------- prefill leg
+    pwl, plabels = prefill_workload()
+    from paper_2608_06849_gb300.workloads import prefill_inputs
+    q, k, v = prefill_inputs(pwl, device="cuda")
+    T = pwl.prefill_len
+    pcache = aoh.Cache(1, pwl.n_q_heads, pwl.n_kv_heads, pwl.d_head, T, pwl.sink, pwl.window, plabels)
+    pout = torch.empty_like(q)
+    Kp = max(3, min(K, args.prefill_steps))
+    for _ in range(max(W, 3)):
+        pcache.reset()
+        pcache.prefill(q, k, v, pout)
+    pcache.check()
+    pev = [torch.cuda.Event(enable_timing=True) for _ in range(Kp + 1)]
+    barrier()
+    pev[0].record(stream)
+    for s in range(Kp):
+        pcache.reset()
+        pcache.prefill(q, k, v, pout)
+        pev[s + 1].record(stream)
+    barrier()
+    clock_info = clocks.stop() if clocks else None
+    pre_ms = max_over_ranks(pev[0].elapsed_time(pev[Kp])) / Kp
+    pcache.check()
+    flops = prefill_flops(pwl, plabels, T)
+    pre_tflops = flops / (pre_ms * 1e-3) / 1e12
+    pcache.close()
+
+    # ---------------- cpu baseline (oracle on a bounded sample), rank 0 only
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = oracle_decode_sample(args.cpu_seconds)
+
+    if rank != 0:
+        return
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    tf_peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    line = {
+        "metric": METRIC,
+        "value": round(dec_us_step, 3),
+        "unit": "us/step",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": round(dec_us_step / 1000.0, 6),
+        "higher_is_better": False,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": f"{wl.name}: B={B} Hq={wl.n_q_heads} Hkv={wl.n_kv_heads} d={D} ctx={T0} "
+                        f"streaming={sum(labels)}/{len(labels)} S={wl.sink} W={wl.window}",
+            "prefill_workload": f"{pwl.name}: T={T} Hq={pwl.n_q_heads} Hkv={pwl.n_kv_heads} d={pwl.d_head} "
+                                f"streaming={sum(plabels)}/{len(plabels)} S={pwl.sink} W={pwl.window}",
+            "l2": "inputs larger than L2 (decode reads a 4.4 GB cache per step; prefill q/k/v 302 MB)",
+            "parallelism": f"replicas x{world}",
+        },
+        "decode": {"us_per_step": round(dec_us_step, 3), "hbm_gbs": round(dec_gbs, 1),
+                   "bytes_per_step": int(avg_bytes), "kernel_us_median": round(statistics.median(per_step_ms) * 1000, 3)},
+        "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                     "frac": round(dec_gbs / hbm_peak, 4), "traffic": traffic_for("decode"),
+                     "peak_note": f"{peak_note} HBM copy bandwidth; kernel: decode split-KV"},
+        "prefill": {"ms": round(pre_ms, 3), "tflops": round(pre_tflops, 2), "flops": flops, "steps": Kp,
+                    "roofline": {"bound": "tensor", "achieved": round(pre_tflops, 2), "peak": tf_peak,
+                                 "unit": "TFLOP/s", "frac": round(pre_tflops / tf_peak, 4),
+                                 "traffic": traffic_for("prefill"),
+                                 "peak_note": f"{peak_note} dense bf16 (burst); time includes the cache append"}},
+        "e2e": {"value": round(e2e_us, 3), "unit": "us/step", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": K,
+        "clocks": clock_info,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+
+
+def traffic_for(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source (else null)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    try:
+        d = json.load(open(p)).get(kernel)
+        if not d:
+            return None
+        from paper_2608_06849_gb300.build import source_digest
+        if d.get("source_digest") != source_digest():
+            return None
+        return d.get("bytes_per_launch")
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------------- reference arm
+
+class OracleDecodeSample:
+    """The float64 oracle on one sequence's decode step at 128K context, for
+    one retrieval and one streaming KV head group; scaled to the full step
+    (16 sequences x 4 retrieval + 4 streaming groups, one pair per scale unit)."""
+
+    def __init__(self):
+        import numpy as np
+
+        from paper_2608_06849_gb300.workloads import randn_bf16
+
+        self.wl, self.labels = decode_workload()
+        D, g, T = self.wl.d_head, self.wl.g, self.wl.prefill_len
+        self.k = randn_bf16((T + 1, 2, D), 9001).float().numpy().astype(np.float64)
+        self.v = randn_bf16((T + 1, 2, D), 9002).float().numpy().astype(np.float64)
+        self.q = randn_bf16((2 * g, D), 9003).float().numpy().astype(np.float64)
+        n_r = len(self.labels) - sum(self.labels)
+        assert n_r == sum(self.labels)
+        self.scale = self.wl.batch * n_r
+
+    def step_us(self):
+        from oracle import attention as oatt
+        t0 = time.perf_counter()
+        oatt.decode_step(self.q, self.k, self.v, [0, 1], self.wl.sink, self.wl.window)
+        return (time.perf_counter() - t0) * 1e6 * self.scale
+
+    def describe(self, reps):
+        return (f"float64 oracle, 1 of {self.wl.batch} sequences x (1 retrieval + 1 streaming) of "
+                f"{len(self.labels)} KV head groups at ctx {self.wl.prefill_len}, median of {reps} reps, "
+                f"scaled x{self.scale}; numpy default BLAS threading")
+
+
+def oracle_decode_sample(budget_s=15.0):
+    s = OracleDecodeSample()
+    s.step_us()
+    vals = []
+    t0 = time.perf_counter()
+    while not vals or time.perf_counter() - t0 < budget_s:
+        vals.append(s.step_us())
+    return {"value": round(statistics.median(vals), 1), "unit": "us/step", "cores": os.cpu_count(),
+            "kind": "oracle", "sample": s.describe(len(vals))}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    s = OracleDecodeSample()
+    for _ in range(args.warmup):
+        s.step_us()
+    vals = [s.step_us() for _ in range(args.steps)]
+    value = sum(vals) / len(vals)
+    wl, labels = s.wl, s.labels
+    line = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": round(value, 1),
+        "unit": "us/step",
+        "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(value / 1000.0, 3),
+        "higher_is_better": False,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"{wl.name}: B={wl.batch} Hq={wl.n_q_heads} Hkv={wl.n_kv_heads} d={wl.d_head} "
+                               f"ctx={wl.prefill_len} streaming={sum(labels)}/{len(labels)} S={wl.sink} W={wl.window}"},
+        "cpu_baseline": {"value": round(value, 1), "unit": "us/step", "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": s.describe(len(vals))},
+        "e2e": {"value": round(value, 1), "unit": "us/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=64)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--prefill-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "native":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

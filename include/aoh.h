@@ -1,0 +1,172 @@
+/*
+ * aoh.h - C ABI of the AoH head-heterogeneous causal attention library
+ * (GB300 / sm_103a).
+ *
+ * The paper (Sec. 5, "Deploying LLMs With AoH") splits the KV heads of every
+ * layer into two kinds:
+ *   retrieval heads keep the full K/V history and run full causal attention;
+ *   streaming heads keep S sink tokens plus the W most recent tokens (a fixed
+ *   per-head cache) and attend only to those ("Chunked-Prefill Stage").
+ * Query heads inherit the label of their KV head (Appendix "GQA Extension").
+ * Each head is computed independently and the outputs sit at their own head
+ * index, which is the concatenation of Eq. 8 (the W_O projection that follows
+ * is outside this library).
+ *
+ * Conventions for every call
+ *   - Element type of q, k, v, out and of the cache is bfloat16 (2 bytes),
+ *     passed as untyped pointers. Accumulation is fp32.
+ *   - All tensors are dense, row-major, and live in device memory of the
+ *     current CUDA device, unless a parameter says otherwise. Each device
+ *     pointer must be 16-byte aligned.
+ *   - Query head h belongs to KV head h / (n_q_heads / n_kv_heads).
+ *   - A key at position j is visible to the query at position i iff j <= i
+ *     and, for a streaming KV head, (j < S or i - j < W): the window counts
+ *     the query's own position.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream). Calls are asynchronous and stream-ordered; calls that use one
+ *     cache must be ordered on one stream (or synchronised by the caller).
+ *   - Every call returns a status and never aborts; on failure
+ *     aoh_last_error() returns a message for the calling thread. Invalid
+ *     arguments are caught on the host before anything is launched.
+ *
+ * Ownership: the caller allocates and frees the KV buffer, the inputs and the
+ * outputs. The handle owns only host state and a small device metadata block
+ * (sequence lengths, split-KV scratch, an error word), allocated by
+ * aoh_cache_init and released by aoh_cache_destroy.
+ */
+#ifndef AOH_H_
+#define AOH_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum aoh_status {
+  AOH_OK = 0,
+  AOH_ERR_INVALID = 1,     /* null pointer, bad shape, misaligned pointer, bad label */
+  AOH_ERR_CAPACITY = 2,    /* buffer too small, or a sequence would pass max_seq   */
+  AOH_ERR_CUDA = 3,        /* a CUDA runtime call failed                           */
+  AOH_ERR_TIMEOUT = 4,     /* a kernel's bounded wait ran out (see aoh_cache_check) */
+  AOH_ERR_UNSUPPORTED = 5, /* d_head or group size outside the compiled kernels    */
+  AOH_ERR_STATE = 6        /* call not valid in the cache's current state          */
+} aoh_status;
+
+/* Labels of a KV head (one uint8 per KV head). */
+#define AOH_RETRIEVAL 0
+#define AOH_STREAMING 1
+
+typedef struct aoh_config {
+  int32_t batch;      /* B: sequences in the cache, >= 1                           */
+  int32_t n_q_heads;  /* Hq, a multiple of n_kv_heads                             */
+  int32_t n_kv_heads; /* Hkv                                                      */
+  int32_t d_head;     /* 64 or 128                                                */
+  int32_t max_seq;    /* tokens a retrieval head can hold per sequence, >= 1      */
+  int32_t sink;       /* S >= 0: sink tokens kept by a streaming head             */
+  int32_t window;     /* W >= 1: recent tokens kept by a streaming head           */
+} aoh_config;
+
+typedef struct aoh_cache aoh_cache; /* opaque handle */
+
+/*
+ * Exact byte size of the KV buffer for `cfg` and `head_labels` [n_kv_heads]:
+ *   B * (n_R * max_seq + n_S * (S + W)) * d_head * 2 (K and V) * 2 (bf16),
+ * n_R / n_S = number of retrieval / streaming KV heads. This is the per-layer
+ * KV memory the paper accounts (Appendix "Details on Baseline Budgets" 32K
+ * KV-memory table; memory columns of Appendix "Additional Efficiency
+ * Results"). Returns 0 if the arguments are invalid (message in
+ * aoh_last_error()). Host only.
+ */
+size_t aoh_cache_bytes(const aoh_config* cfg, const uint8_t* head_labels);
+
+/*
+ * Bind a caller-owned device buffer as an empty KV cache (all lengths 0).
+ *   cfg          shape and streaming parameters (copied).
+ *   head_labels  host array [n_kv_heads] of AOH_RETRIEVAL / AOH_STREAMING
+ *                (copied).
+ *   kv_buffer    device pointer, 256-byte aligned, at least
+ *                aoh_cache_bytes(cfg, head_labels) bytes; its contents need
+ *                not be initialised. Not freed by the library.
+ *   out          receives the handle.
+ * Layout of kv_buffer: first one region per (sequence b, retrieval head) in
+ * order b-major, retrieval heads in increasing KV-head index; then one region
+ * per (b, streaming head) in the same order. A region is K[capacity][d_head]
+ * followed by V[capacity][d_head], capacity = max_seq (retrieval) or S + W
+ * (streaming). A retrieval head stores position p at row p. A streaming head
+ * stores position p < S at row p and position p >= S at row
+ * S + (p - S) mod W (a ring of W rows after the sinks). aoh_cache_region()
+ * returns the offsets.
+ * Synchronises the device once (metadata upload). Errors: INVALID, CAPACITY,
+ * UNSUPPORTED, CUDA.
+ */
+aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
+                          size_t kv_buffer_bytes, aoh_cache** out);
+
+/*
+ * Causal prefill of an empty cache (the paper's prefill stage, Sec. 5 and the
+ * inference-phase appendix; every streaming query uses the per-token
+ * sink + window rule above).
+ *   q    [B][T][n_q_heads][d_head]
+ *   k, v [B][T][n_kv_heads][d_head]
+ *   T    padded sequence length, 1 <= T <= max_seq.
+ *   seq_lens  host array [B] of lengths 1..T, or NULL (all T). Rows at or
+ *             past seq_lens[b] are not read and their outputs not written.
+ *   out  [B][T][n_q_heads][d_head], or NULL to only fill the cache.
+ * Writes K/V of every position into the retrieval regions and the sinks plus
+ * the last W positions into the streaming regions, then sets the lengths.
+ * Errors: INVALID, CAPACITY (T > max_seq), STATE (cache not empty), CUDA.
+ */
+aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T,
+                       const int32_t* seq_lens, aoh_cache* cache, void* out, void* stream);
+
+/*
+ * One decode step for every sequence (Sec. 5 "Decode Stage", Eq. 8): the new
+ * token of sequence b sits at position t = len(b); its K/V are appended (the
+ * streaming ring overwrites the position that leaves the window) and its
+ * query attends over positions visible to it; len(b) becomes t + 1.
+ *   q            [B][n_q_heads][d_head]
+ *   k_new, v_new [B][n_kv_heads][d_head]
+ *   out          [B][n_q_heads][d_head]
+ * The lengths advance on the device as well as in the handle, so consecutive
+ * steps need no host work between them. Errors: INVALID, CAPACITY (a
+ * retrieval head would pass max_seq; nothing is launched), CUDA.
+ */
+aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,
+                           void* out, void* stream);
+
+/* Copy the host-side lengths (tokens held per sequence) into lens_out [B]. */
+aoh_status aoh_cache_lens(const aoh_cache* cache, int32_t* lens_out);
+
+/*
+ * Byte offsets (from kv_buffer) of the K and V rows of sequence b, KV head h,
+ * and that region's capacity in rows. Host only; for inspection and tests.
+ */
+aoh_status aoh_cache_region(const aoh_cache* cache, int32_t b, int32_t kv_head, size_t* k_offset,
+                            size_t* v_offset, int32_t* capacity);
+
+/* Mark every sequence empty again (host and device lengths), stream-ordered. */
+aoh_status aoh_cache_reset(aoh_cache* cache, void* stream);
+
+/*
+ * Synchronise `stream` and read the device error word that kernels set when
+ * a bounded wait runs out. Returns AOH_OK, AOH_ERR_TIMEOUT (and clears the
+ * word) or AOH_ERR_CUDA.
+ */
+aoh_status aoh_cache_check(aoh_cache* cache, void* stream);
+
+/* Release the handle and its device metadata (not the KV buffer). NULL is a no-op. */
+void aoh_cache_destroy(aoh_cache* cache);
+
+/* Message of the last failed call on this thread ("" if none). */
+const char* aoh_last_error(void);
+
+/* Library ABI version (major * 100 + minor). */
+int32_t aoh_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AOH_H_ */

@@ -1,0 +1,219 @@
+"""ctypes binding of ``libaoh.so`` (the C ABI in ``include/aoh.h``).
+
+Argument marshalling only: every step of the attention path runs in the
+library's CUDA kernels. The functions carry the C names; torch tensors are
+passed as raw device pointers plus the current CUDA stream. There is no
+fallback: if the library is missing or fails to load, every call raises.
+
+``Cache`` is a small convenience owner of a KV buffer (a torch uint8 device
+tensor) and its handle.
+"""
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libaoh.so")
+
+AOH_OK = 0
+STATUS_NAMES = {0: "OK", 1: "INVALID", 2: "CAPACITY", 3: "CUDA", 4: "TIMEOUT", 5: "UNSUPPORTED", 6: "STATE"}
+RETRIEVAL = 0
+STREAMING = 1
+
+EXPORTS = [
+    "aoh_cache_bytes",
+    "aoh_cache_init",
+    "aoh_prefill",
+    "aoh_decode_step",
+    "aoh_cache_lens",
+    "aoh_cache_region",
+    "aoh_cache_reset",
+    "aoh_cache_check",
+    "aoh_cache_destroy",
+    "aoh_last_error",
+    "aoh_version",
+]
+
+
+class AohError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"aoh status {STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+class aoh_config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("batch", "n_q_heads", "n_kv_heads", "d_head", "max_seq", "sink", "window")]
+
+
+_lib = None
+
+
+def load():
+    """Load ``libaoh.so`` once; raise if it is absent (no CPU fallback)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2608_06849_gb300.build.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P = ctypes.c_void_p
+    i32 = ctypes.c_int32
+    cfgp = ctypes.POINTER(aoh_config)
+    u8p = ctypes.POINTER(ctypes.c_uint8)
+    i32p = ctypes.POINTER(ctypes.c_int32)
+    szp = ctypes.POINTER(ctypes.c_size_t)
+    sig = {
+        "aoh_cache_bytes": (ctypes.c_size_t, [cfgp, u8p]),
+        "aoh_cache_init": (i32, [cfgp, u8p, P, ctypes.c_size_t, ctypes.POINTER(P)]),
+        "aoh_prefill": (i32, [P, P, P, i32, i32p, P, P, P]),
+        "aoh_decode_step": (i32, [P, P, P, P, P, P]),
+        "aoh_cache_lens": (i32, [P, i32p]),
+        "aoh_cache_region": (i32, [P, i32, i32, szp, szp, i32p]),
+        "aoh_cache_reset": (i32, [P, P]),
+        "aoh_cache_check": (i32, [P, P]),
+        "aoh_cache_destroy": (None, [P]),
+        "aoh_last_error": (ctypes.c_char_p, []),
+        "aoh_version": (i32, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(status):
+    if status != AOH_OK:
+        raise AohError(status, load().aoh_last_error().decode())
+
+
+def _labels_arr(labels):
+    return (ctypes.c_uint8 * len(labels))(*[int(x) for x in labels])
+
+
+def make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window):
+    return aoh_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window)
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t, name, dtype=torch.bfloat16):
+    if t is None:
+        return None
+    if not t.is_cuda or t.dtype != dtype or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous {dtype} CUDA tensor")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+# ----------------------------------------------------------------- C names
+
+def aoh_version():
+    return load().aoh_version()
+
+
+def aoh_cache_bytes(cfg, labels):
+    n = load().aoh_cache_bytes(ctypes.byref(cfg), _labels_arr(labels))
+    if n == 0:
+        raise AohError(1, load().aoh_last_error().decode())
+    return n
+
+
+def aoh_cache_init(cfg, labels, kv_buffer):
+    """kv_buffer: a CUDA uint8 tensor of at least aoh_cache_bytes() bytes."""
+    h = ctypes.c_void_p()
+    _check(load().aoh_cache_init(ctypes.byref(cfg), _labels_arr(labels), _ptr(kv_buffer, "kv_buffer", torch.uint8),
+                                 kv_buffer.numel(), ctypes.byref(h)))
+    return h
+
+
+def aoh_prefill(q, k, v, T, seq_lens, cache, out, stream=None):
+    lens = None if seq_lens is None else (ctypes.c_int32 * len(seq_lens))(*[int(x) for x in seq_lens])
+    _check(load().aoh_prefill(_ptr(q, "q"), _ptr(k, "k"), _ptr(v, "v"), int(T), lens, cache,
+                              _ptr(out, "out"), _stream_ptr(stream)))
+
+
+def aoh_decode_step(q, k_new, v_new, cache, out, stream=None):
+    _check(load().aoh_decode_step(_ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), cache,
+                                  _ptr(out, "out"), _stream_ptr(stream)))
+
+
+def aoh_cache_lens(cache, batch):
+    arr = (ctypes.c_int32 * batch)()
+    _check(load().aoh_cache_lens(cache, arr))
+    return list(arr)
+
+
+def aoh_cache_region(cache, b, kv_head):
+    ko, vo, cap = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_int32()
+    _check(load().aoh_cache_region(cache, int(b), int(kv_head), ctypes.byref(ko), ctypes.byref(vo),
+                                   ctypes.byref(cap)))
+    return ko.value, vo.value, cap.value
+
+
+def aoh_cache_reset(cache, stream=None):
+    _check(load().aoh_cache_reset(cache, _stream_ptr(stream)))
+
+
+def aoh_cache_check(cache, stream=None):
+    _check(load().aoh_cache_check(cache, _stream_ptr(stream)))
+
+
+def aoh_cache_destroy(cache):
+    load().aoh_cache_destroy(cache)
+
+
+# ------------------------------------------------------------- convenience
+
+class Cache:
+    """A KV buffer on the current CUDA device plus its library handle."""
+
+    def __init__(self, batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, labels, device=None):
+        self.cfg = make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window)
+        self.labels = [int(x) for x in labels]
+        self.nbytes = aoh_cache_bytes(self.cfg, self.labels)
+        self.buffer = torch.empty(self.nbytes, dtype=torch.uint8, device=device or "cuda")
+        self.handle = aoh_cache_init(self.cfg, self.labels, self.buffer)
+        self.batch, self.n_q_heads, self.n_kv_heads, self.d_head = batch, n_q_heads, n_kv_heads, d_head
+        self.max_seq, self.sink, self.window = max_seq, sink, window
+
+    def prefill(self, q, k, v, out=None, seq_lens=None, stream=None):
+        aoh_prefill(q, k, v, k.shape[1], seq_lens, self.handle, out, stream)
+
+    def decode_step(self, q, k_new, v_new, out, stream=None):
+        aoh_decode_step(q, k_new, v_new, self.handle, out, stream)
+
+    def lens(self):
+        return aoh_cache_lens(self.handle, self.batch)
+
+    def region(self, b, kv_head):
+        """(K rows, V rows) of (b, kv_head) as bf16 views [capacity, d_head] of the buffer."""
+        ko, vo, cap = aoh_cache_region(self.handle, b, kv_head)
+        nb = cap * self.d_head * 2
+        kr = self.buffer[ko:ko + nb].view(torch.bfloat16).view(cap, self.d_head)
+        vr = self.buffer[vo:vo + nb].view(torch.bfloat16).view(cap, self.d_head)
+        return kr, vr
+
+    def reset(self, stream=None):
+        aoh_cache_reset(self.handle, stream)
+
+    def check(self, stream=None):
+        aoh_cache_check(self.handle, stream)
+
+    def close(self):
+        if getattr(self, "handle", None):
+            aoh_cache_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,324 @@
+// Host runtime behind include/aoh.h: argument validation, cache layout,
+// split-KV scheduling and kernel launches on the caller's stream.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <algorithm>
+#include <string>
+#include <vector>
+
+#include "../../include/aoh.h"
+#include "internal.h"
+
+using namespace aoh;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+aoh_status fail(aoh_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+aoh_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(AOH_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Validates cfg + labels; fills n_r / n_s. Returns AOH_OK or an error.
+aoh_status check_config(const aoh_config* cfg, const uint8_t* labels, int* n_r, int* n_s) {
+  if (!cfg) return fail(AOH_ERR_INVALID, "cfg is NULL");
+  if (!labels) return fail(AOH_ERR_INVALID, "head_labels is NULL");
+  const aoh_config& c = *cfg;
+  if (c.batch < 1 || c.n_q_heads < 1 || c.n_kv_heads < 1 || c.max_seq < 1)
+    return fail(AOH_ERR_INVALID, "batch, n_q_heads, n_kv_heads and max_seq must be >= 1");
+  if (c.n_kv_heads > kMaxKvHeads) return fail(AOH_ERR_UNSUPPORTED, "n_kv_heads > %d", kMaxKvHeads);
+  if (c.n_q_heads % c.n_kv_heads) return fail(AOH_ERR_INVALID, "n_q_heads must be a multiple of n_kv_heads");
+  if (c.d_head != 64 && c.d_head != 128) return fail(AOH_ERR_UNSUPPORTED, "d_head must be 64 or 128");
+  if (c.sink < 0 || c.window < 1) return fail(AOH_ERR_INVALID, "need sink >= 0 and window >= 1");
+  int r = 0, s = 0;
+  for (int h = 0; h < c.n_kv_heads; ++h) {
+    if (labels[h] == AOH_RETRIEVAL)
+      ++r;
+    else if (labels[h] == AOH_STREAMING)
+      ++s;
+    else
+      return fail(AOH_ERR_INVALID, "head_labels[%d] = %d is neither retrieval (0) nor streaming (1)", h,
+                  (int)labels[h]);
+  }
+  *n_r = r;
+  *n_s = s;
+  return AOH_OK;
+}
+
+size_t bytes_for(const aoh_config& c, int n_r, int n_s) {
+  const size_t tokens = (size_t)n_r * c.max_seq + (size_t)n_s * (size_t)(c.sink + c.window);
+  return (size_t)c.batch * tokens * c.d_head * 2 * 2;
+}
+
+}  // namespace
+
+struct aoh_cache {
+  aoh_config cfg;
+  CacheGeom geom;
+  std::vector<uint8_t> labels;
+  void* kv = nullptr;
+  size_t kv_bytes = 0;
+  std::vector<int32_t> lens;  // host mirror of the device lengths
+  int device = 0;
+  int num_sms = 0;
+  int split_stride = 1;
+  // device metadata (one allocation)
+  void* meta = nullptr;
+  int32_t* d_lens = nullptr;
+  uint32_t* d_counters = nullptr;
+  uint32_t* d_done = nullptr;
+  uint32_t* d_err = nullptr;
+  float* d_partials = nullptr;
+};
+
+extern "C" {
+
+int32_t aoh_version(void) { return 100; }
+
+const char* aoh_last_error(void) { return g_last_error.c_str(); }
+
+size_t aoh_cache_bytes(const aoh_config* cfg, const uint8_t* head_labels) {
+  int n_r, n_s;
+  if (check_config(cfg, head_labels, &n_r, &n_s) != AOH_OK) return 0;
+  return bytes_for(*cfg, n_r, n_s);
+}
+
+aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
+                          size_t kv_buffer_bytes, aoh_cache** out) {
+  if (!out) return fail(AOH_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  int n_r, n_s;
+  aoh_status st = check_config(cfg, head_labels, &n_r, &n_s);
+  if (st != AOH_OK) return st;
+  const aoh_config& c = *cfg;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  if (!decode_supported(c.d_head, G) || !prefill_supported(c.d_head, G))
+    return fail(AOH_ERR_UNSUPPORTED, "group size %d with d_head %d is not compiled", G, c.d_head);
+  if (!kv_buffer) return fail(AOH_ERR_INVALID, "kv_buffer is NULL");
+  if (!aligned(kv_buffer, 256)) return fail(AOH_ERR_INVALID, "kv_buffer must be 256-byte aligned");
+  const size_t need = bytes_for(c, n_r, n_s);
+  if (kv_buffer_bytes < need)
+    return fail(AOH_ERR_CAPACITY, "kv_buffer has %zu bytes, the cache needs %zu", kv_buffer_bytes, need);
+
+  aoh_cache* h = new aoh_cache();
+  h->cfg = c;
+  h->labels.assign(head_labels, head_labels + c.n_kv_heads);
+  h->kv = kv_buffer;
+  h->kv_bytes = need;
+  h->lens.assign(c.batch, 0);
+  CacheGeom& g = h->geom;
+  g.B = c.batch;
+  g.Hq = c.n_q_heads;
+  g.Hkv = c.n_kv_heads;
+  g.D = c.d_head;
+  g.G = G;
+  g.max_seq = c.max_seq;
+  g.S = c.sink;
+  g.W = c.window;
+  g.n_r = n_r;
+  g.n_s = n_s;
+  int ir = 0, is = 0;
+  for (int k = 0; k < c.n_kv_heads; ++k) {
+    g.kind[k] = head_labels[k];
+    if (head_labels[k] == AOH_RETRIEVAL) {
+      g.idx[k] = (uint8_t)ir;
+      g.r_head[ir++] = (uint8_t)k;
+    } else {
+      g.idx[k] = (uint8_t)is;
+      g.s_head[is++] = (uint8_t)k;
+    }
+  }
+
+  cudaError_t e = cudaGetDevice(&h->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+  if (e != cudaSuccess) {
+    delete h;
+    return cuda_fail(e, "cudaGetDevice");
+  }
+  const int longest = std::max(c.max_seq, c.sink + c.window);
+  h->split_stride = std::min(kMaxSplits, std::max(1, (longest + 511) / 512));
+  const size_t n_lens = ((size_t)c.batch + 63) / 64 * 64;
+  const size_t n_cnt = ((size_t)c.batch * c.n_kv_heads + 63) / 64 * 64;
+  const size_t n_part = (size_t)c.batch * c.n_kv_heads * h->split_stride * G * (c.d_head + 2);
+  const size_t meta_bytes = (n_lens + n_cnt + 64) * 4 + n_part * 4;
+  e = cudaMalloc(&h->meta, meta_bytes);
+  if (e == cudaSuccess) e = cudaMemset(h->meta, 0, meta_bytes);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    if (h->meta) cudaFree(h->meta);
+    delete h;
+    return cuda_fail(e, "metadata allocation");
+  }
+  uint32_t* base = static_cast<uint32_t*>(h->meta);
+  h->d_lens = reinterpret_cast<int32_t*>(base);
+  h->d_counters = base + n_lens;
+  h->d_done = h->d_counters + n_cnt;
+  h->d_err = h->d_done + 32;
+  h->d_partials = reinterpret_cast<float*>(base + n_lens + n_cnt + 64);
+  *out = h;
+  return AOH_OK;
+}
+
+void aoh_cache_destroy(aoh_cache* cache) {
+  if (!cache) return;
+  if (cache->meta) cudaFree(cache->meta);
+  delete cache;
+}
+
+aoh_status aoh_cache_lens(const aoh_cache* cache, int32_t* lens_out) {
+  if (!cache || !lens_out) return fail(AOH_ERR_INVALID, "NULL argument");
+  std::copy(cache->lens.begin(), cache->lens.end(), lens_out);
+  return AOH_OK;
+}
+
+aoh_status aoh_cache_region(const aoh_cache* cache, int32_t b, int32_t kv_head, size_t* k_offset,
+                            size_t* v_offset, int32_t* capacity) {
+  if (!cache || !k_offset || !v_offset || !capacity) return fail(AOH_ERR_INVALID, "NULL argument");
+  const CacheGeom& g = cache->geom;
+  if (b < 0 || b >= g.B || kv_head < 0 || kv_head >= g.Hkv) return fail(AOH_ERR_INVALID, "b or kv_head out of range");
+  const size_t elem = g.region(b, kv_head);
+  *capacity = g.capacity(kv_head);
+  *k_offset = elem * 2;
+  *v_offset = (elem + (size_t)(*capacity) * g.D) * 2;
+  return AOH_OK;
+}
+
+aoh_status aoh_cache_reset(aoh_cache* cache, void* stream) {
+  if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
+  std::fill(cache->lens.begin(), cache->lens.end(), 0);
+  cudaError_t e = cudaMemsetAsync(cache->d_lens, 0, sizeof(int32_t) * cache->geom.B, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  return AOH_OK;
+}
+
+aoh_status aoh_cache_check(aoh_cache* cache, void* stream) {
+  if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  uint32_t err = 0;
+  e = cudaMemcpy(&err, cache->d_err, sizeof(err), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+  if (err) {
+    const uint32_t zero = 0;
+    cudaMemcpy(cache->d_err, &zero, sizeof(zero), cudaMemcpyHostToDevice);
+    return fail(AOH_ERR_TIMEOUT, "a kernel's bounded wait ran out (error word 0x%x)", err);
+  }
+  return AOH_OK;
+}
+
+aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, const int32_t* seq_lens,
+                       aoh_cache* cache, void* out, void* stream) {
+  if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
+  if (!k || !v) return fail(AOH_ERR_INVALID, "k and v must not be NULL");
+  if (out && !q) return fail(AOH_ERR_INVALID, "q must not be NULL when out is given");
+  if (!aligned(k, 16) || !aligned(v, 16) || (q && !aligned(q, 16)) || (out && !aligned(out, 16)))
+    return fail(AOH_ERR_INVALID, "q, k, v and out must be 16-byte aligned");
+  const CacheGeom& g = cache->geom;
+  if (T < 1) return fail(AOH_ERR_INVALID, "T must be >= 1");
+  if (T > g.max_seq) return fail(AOH_ERR_CAPACITY, "T = %d exceeds max_seq = %d", T, g.max_seq);
+  for (int b = 0; b < g.B; ++b)
+    if (cache->lens[b] != 0) return fail(AOH_ERR_STATE, "prefill needs an empty cache (sequence %d holds %d tokens)", b, cache->lens[b]);
+  std::vector<int32_t> lens(g.B, T);
+  if (seq_lens) {
+    for (int b = 0; b < g.B; ++b) {
+      if (seq_lens[b] < 1 || seq_lens[b] > T)
+        return fail(AOH_ERR_INVALID, "seq_lens[%d] = %d is outside [1, T]", b, seq_lens[b]);
+      lens[b] = seq_lens[b];
+    }
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(cache->d_lens, lens.data(), sizeof(int32_t) * g.B, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(lens)");
+
+  AppendArgs ap;
+  ap.geom = g;
+  ap.k = k;
+  ap.v = v;
+  ap.kv = cache->kv;
+  ap.lens = cache->d_lens;
+  ap.T = T;
+  e = launch_append(ap, s);
+  if (e != cudaSuccess) return cuda_fail(e, "append kernel launch");
+
+  if (out) {
+    PrefillArgs pa;
+    pa.geom = g;
+    pa.q = q;
+    pa.k = k;
+    pa.v = v;
+    pa.out = out;
+    pa.lens = cache->d_lens;
+    pa.T = T;
+    pa.scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
+    pa.work = nullptr;
+    pa.n_work = 0;
+    pa.err = cache->d_err;
+    e = launch_prefill(pa, s);
+    if (e != cudaSuccess) return cuda_fail(e, "prefill kernel launch");
+  }
+  cache->lens = lens;
+  return AOH_OK;
+}
+
+aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, aoh_cache* cache, void* out,
+                           void* stream) {
+  if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
+  if (!q || !k_new || !v_new || !out) return fail(AOH_ERR_INVALID, "q, k_new, v_new and out must not be NULL");
+  if (!aligned(q, 16) || !aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(out, 16))
+    return fail(AOH_ERR_INVALID, "q, k_new, v_new and out must be 16-byte aligned");
+  const CacheGeom& g = cache->geom;
+  int maxlen = 0;
+  for (int b = 0; b < g.B; ++b) {
+    if (g.n_r > 0 && cache->lens[b] + 1 > g.max_seq)
+      return fail(AOH_ERR_CAPACITY, "sequence %d holds %d tokens; max_seq is %d", b, cache->lens[b], g.max_seq);
+    maxlen = std::max(maxlen, cache->lens[b] + 1);
+  }
+  // Split-KV schedule: rows per split chosen so the launch holds a few waves
+  // of CTAs; streaming heads get splits of about the same size.
+  const int win = std::min(maxlen, g.S + g.W);
+  double total = 0;
+  for (int b = 0; b < g.B; ++b)
+    total += (double)g.n_r * (cache->lens[b] + 1) + (double)g.n_s * std::min(cache->lens[b] + 1, g.S + g.W);
+  const double target_ctas = (double)cache->num_sms * 2 * 4;
+  const int chunk = std::max(512, (int)ceil(total / target_ctas));
+  const int ns_r = g.n_r ? std::min(cache->split_stride, std::max(1, (maxlen + chunk - 1) / chunk)) : 0;
+  const int ns_s = g.n_s ? std::min(cache->split_stride, std::max(1, (win + chunk - 1) / chunk)) : 0;
+
+  DecodeArgs a;
+  a.geom = g;
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.out = out;
+  a.kv = cache->kv;
+  a.lens = cache->d_lens;
+  a.partials = cache->d_partials;
+  a.counters = cache->d_counters;
+  a.done = cache->d_done;
+  a.err = cache->d_err;
+  a.ns_r = ns_r;
+  a.ns_s = ns_s;
+  a.split_stride = cache->split_stride;
+  a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
+  const int n_ctas = g.B * (g.n_r * ns_r + g.n_s * ns_s);
+  cudaError_t e = launch_decode(a, n_ctas, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");
+  for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
+  return AOH_OK;
+}
+
+}  // extern "C"

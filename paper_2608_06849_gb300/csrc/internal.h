@@ -1,0 +1,85 @@
+// Host-side declarations shared by the translation units of libaoh.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace aoh {
+
+constexpr int kMaxKvHeads = 64;
+constexpr int kMaxSplits = 64;  // split-KV partials per (sequence, KV head)
+
+// Cache geometry as the kernels see it. Offsets are in bf16 elements from the
+// cache base; see include/aoh.h for the layout.
+struct CacheGeom {
+  int B, Hq, Hkv, D, G;
+  int max_seq, S, W;
+  int n_r, n_s;
+  // kind[h] = 0 retrieval / 1 streaming; idx[h] = index among heads of its kind
+  uint8_t kind[kMaxKvHeads];
+  uint8_t idx[kMaxKvHeads];
+  uint8_t r_head[kMaxKvHeads];  // i-th retrieval head -> KV head
+  uint8_t s_head[kMaxKvHeads];  // i-th streaming head -> KV head
+
+  __host__ __device__ size_t r_region(int b, int i) const {
+    return (size_t)(b * n_r + i) * 2 * (size_t)max_seq * D;
+  }
+  __host__ __device__ size_t s_region(int b, int i) const {
+    return (size_t)B * n_r * 2 * (size_t)max_seq * D + (size_t)(b * n_s + i) * 2 * (size_t)(S + W) * D;
+  }
+  // K region start of (b, kv head); V follows after capacity rows.
+  __host__ __device__ size_t region(int b, int h) const {
+    return kind[h] ? s_region(b, idx[h]) : r_region(b, idx[h]);
+  }
+  __host__ __device__ int capacity(int h) const { return kind[h] ? S + W : max_seq; }
+};
+
+struct DecodeArgs {
+  CacheGeom geom;
+  const void* q;      // [B][Hq][D]
+  const void* k_new;  // [B][Hkv][D]
+  const void* v_new;
+  void* out;          // [B][Hq][D]
+  void* kv;           // cache base
+  int32_t* lens;      // [B] tokens held before this step (device)
+  float* partials;    // [B][Hkv][split_stride][G][D + 2]
+  uint32_t* counters; // [B][Hkv] split arrivals
+  uint32_t* done;     // CTAs finished in this launch
+  uint32_t* err;      // error word
+  int ns_r, ns_s;     // splits per retrieval / streaming head
+  int split_stride;   // partial slots per (b, head) in `partials`, >= ns_r, ns_s
+  float scale_log2;   // log2(e) / sqrt(D)
+};
+
+struct AppendArgs {
+  CacheGeom geom;
+  const void* k;  // [B][T][Hkv][D]
+  const void* v;
+  void* kv;
+  const int32_t* lens;  // device [B]
+  int T;
+};
+
+struct PrefillArgs {
+  CacheGeom geom;
+  const void* q;  // [B][T][Hq][D]
+  const void* k;  // [B][T][Hkv][D]
+  const void* v;
+  void* out;      // [B][T][Hq][D]
+  const int32_t* lens;  // device [B]
+  int T;
+  float scale_log2;
+  const int4* work;  // work items
+  int n_work;
+  uint32_t* err;
+};
+
+// Launchers (return the launch's cudaError_t).
+cudaError_t launch_decode(const DecodeArgs& a, int n_ctas, cudaStream_t s);
+cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t s);
+bool decode_supported(int D, int G);
+bool prefill_supported(int D, int G);
+
+}  // namespace aoh

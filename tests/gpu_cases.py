@@ -1,0 +1,118 @@
+"""Shared helpers of the GPU parity tests: run a case through the C ABI and
+compare it with the oracle on the same bf16 inputs."""
+
+import numpy as np
+import torch
+
+from oracle import attention as oatt
+from paper_2608_06849_gb300 import aoh
+from paper_2608_06849_gb300 import build as aoh_build
+from paper_2608_06849_gb300.workloads import Workload, decode_inputs, prefill_inputs
+
+MAX_ABS = 1e-2    # the bound on max |err| against the oracle
+MEAN_ABS = 1e-3   # the bound on mean |err|
+
+_built = False
+
+
+def ensure_lib():
+    global _built
+    if not _built:
+        aoh_build.build()
+        aoh.load()
+        _built = True
+
+
+def f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def assert_matches(got, want, what=""):
+    """max/mean absolute bounds, plus an elementwise bound of two bf16 ulps of
+    the exact value (the output is rounded to bf16 once) + 1e-3."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    assert got.shape == want.shape, (got.shape, want.shape)
+    assert np.isfinite(got).all(), f"{what}: non-finite output"
+    err = np.abs(got - want)
+    assert err.max() <= MAX_ABS, f"{what}: max |err| {err.max():.3e}"
+    assert err.mean() <= MEAN_ABS, f"{what}: mean |err| {err.mean():.3e}"
+    bound = np.abs(want) * 2.0 ** -8 + 1e-3
+    bad = err > bound
+    assert not bad.any(), f"{what}: {bad.sum()} elements beyond 2 ulp, worst {err[bad].max():.3e}"
+    return err.max(), err.mean()
+
+
+def check_cache_image(cache, k, v, lens, labels, S, W):
+    """Bit-exact: retrieval rows 0..len-1 hold K/V of positions 0..len-1;
+    streaming rows hold the sink and ring image the oracle's slot model gives."""
+    for b in range(cache.batch):
+        L = lens[b]
+        for h in range(cache.n_kv_heads):
+            kr, vr = cache.region(b, h)
+            kseq = k[b, :L, h]
+            vseq = v[b, :L, h]
+            if labels[h] == aoh.RETRIEVAL:
+                assert torch.equal(kr[:L].cpu(), kseq.cpu()), (b, h)
+                assert torch.equal(vr[:L].cpu(), vseq.cpu()), (b, h)
+            else:
+                held = oatt.streaming_slots_after(L - 1, S, W)
+                slots = sorted(held)
+                pos = [held[s] for s in slots]
+                assert torch.equal(kr[slots].cpu(), kseq[pos].cpu()), (b, h)
+                assert torch.equal(vr[slots].cpu(), vseq[pos].cpu()), (b, h)
+
+
+def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink_scale=8.0, seed=0,
+             check_prefill_out=True, peaky=1.0, rows=None):
+    """Prefill (+ decode steps) on the GPU; every output compared with the oracle."""
+    ensure_lib()
+    wl = Workload("case", B, Hq, Hkv, d, T, decode_steps, S, W, sum(labels), seed=seed, sink_scale=sink_scale)
+    q, k, v = prefill_inputs(wl, device="cuda")
+    if peaky != 1.0:
+        k = (k.float() * peaky).to(torch.bfloat16)
+    lens = list(seq_lens) if seq_lens is not None else [T] * B
+    cache = aoh.Cache(B, Hq, Hkv, d, T + decode_steps, S, W, labels)
+    out = torch.full_like(q, float("nan"))
+    cache.prefill(q, k, v, out if check_prefill_out else None, seq_lens)
+    torch.cuda.synchronize()
+    cache.check()
+    assert cache.lens() == lens
+    qn, kn, vn = f64(q), f64(k), f64(v)
+    results = {}
+    if check_prefill_out:
+        for b in range(B):
+            r = np.arange(lens[b]) if rows is None else np.asarray([x for x in rows if x < lens[b]])
+            want = oatt.prefill(qn[b, :lens[b]], kn[b, :lens[b]], vn[b, :lens[b]], labels, S, W, rows=r)
+            results[("prefill", b)] = assert_matches(f64(out[b, r]), want, f"prefill b={b}")
+    check_cache_image(cache, k, v, lens, labels, S, W)
+
+    kall = [kn[b, :lens[b]] for b in range(B)]
+    vall = [vn[b, :lens[b]] for b in range(B)]
+    kseq_t = [k[b, :lens[b]] for b in range(B)]
+    vseq_t = [v[b, :lens[b]] for b in range(B)]
+    for step in range(decode_steps):
+        dq, dk, dv = decode_inputs(wl, step, device="cuda")
+        dout = torch.full_like(dq, float("nan"))
+        cache.decode_step(dq, dk, dv, dout)
+        torch.cuda.synchronize()
+        dqn, dkn, dvn = f64(dq), f64(dk), f64(dv)
+        for b in range(B):
+            kall[b] = np.concatenate([kall[b], dkn[b][None]], axis=0)
+            vall[b] = np.concatenate([vall[b], dvn[b][None]], axis=0)
+            kseq_t[b] = torch.cat([kseq_t[b], dk[b][None]], dim=0)
+            vseq_t[b] = torch.cat([vseq_t[b], dv[b][None]], dim=0)
+            want = oatt.decode_step(dqn[b], kall[b], vall[b], labels, S, W)
+            results[("decode", step, b)] = assert_matches(f64(dout[b]), want, f"decode step={step} b={b}")
+    cache.check()
+    if decode_steps:
+        new_lens = [L + decode_steps for L in lens]
+        assert cache.lens() == new_lens
+        kpad = torch.zeros(B, max(new_lens), Hkv, d, dtype=torch.bfloat16)
+        vpad = torch.zeros_like(kpad)
+        for b in range(B):
+            kpad[b, :new_lens[b]] = kseq_t[b].cpu()
+            vpad[b, :new_lens[b]] = vseq_t[b].cpu()
+        check_cache_image(cache, kpad, vpad, new_lens, labels, S, W)
+    cache.close()
+    return results

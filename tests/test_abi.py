@@ -1,0 +1,108 @@
+"""The C-ABI library loads and exports every symbol include/aoh.h declares;
+host-only calls (byte count, argument validation) behave as documented.
+No compute call is made here, so these run without a GPU."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from oracle import kv_memory as kvm
+from paper_2608_06849_gb300 import aoh
+from paper_2608_06849_gb300 import build as aoh_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "aoh.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    aoh_build.build()
+    return aoh.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"\b(aoh_[a-z_]+)\s*\(", text)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ["aoh_cache_bytes", "aoh_cache_init", "aoh_prefill", "aoh_decode_step"]:
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(declared_functions()) <= set(aoh.EXPORTS) | set(declared_functions())
+    assert sorted(aoh.EXPORTS) == declared_functions()
+
+
+def test_version(lib):
+    assert aoh.aoh_version() == 100
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,d,max_seq,S,W,labels", [
+    (1, 8, 2, 64, 1056, 16, 128, [0, 1]),
+    (1, 28, 4, 128, 32768, 128, 2048, [1, 1, 0, 0]),
+    (16, 32, 8, 128, 131136, 128, 4096, [1, 0, 0, 1, 1, 0, 0, 1]),
+    (3, 4, 4, 64, 100, 0, 1, [1, 1, 1, 1]),
+    (2, 4, 2, 128, 7, 5, 9, [0, 0]),
+])
+def test_cache_bytes_matches_formula(lib, B, Hq, Hkv, d, max_seq, S, W, labels):
+    cfg = aoh.make_config(B, Hq, Hkv, d, max_seq, S, W)
+    n_s = sum(labels)
+    want = kvm.kv_cache_bytes(B, Hkv - n_s, n_s, max_seq, S, W, d)
+    assert aoh.aoh_cache_bytes(cfg, labels) == want
+
+
+def test_qwen25_stack_bytes(lib):
+    """28 layers of the Qwen2.5-7B-shaped 256K workload, 2 of 4 KV heads streaming."""
+    cfg = aoh.make_config(1, 28, 4, 128, 262144 + 128, 128, 4096)
+    per_layer = aoh.aoh_cache_bytes(cfg, [0, 1, 1, 0])
+    assert 28 * per_layer == 28 * (2 * 262272 + 2 * 4224) * 128 * 4
+    full = aoh.aoh_cache_bytes(cfg, [0, 0, 0, 0])
+    assert full / per_layer > 1.96
+
+
+@pytest.mark.parametrize("bad", [
+    dict(batch=0), dict(n_q_heads=6, n_kv_heads=4), dict(d_head=96), dict(window=0), dict(sink=-1),
+    dict(max_seq=0),
+])
+def test_invalid_config_rejected_on_host(lib, bad):
+    args = dict(batch=1, n_q_heads=8, n_kv_heads=2, d_head=64, max_seq=64, sink=4, window=8)
+    args.update(bad)
+    cfg = aoh.make_config(**args)
+    n = lib.aoh_cache_bytes(ctypes.byref(cfg), (ctypes.c_uint8 * 4)(0, 1, 0, 1))
+    assert n == 0
+    assert lib.aoh_last_error().decode() != ""
+
+
+def test_bad_label_rejected(lib):
+    cfg = aoh.make_config(1, 8, 2, 64, 64, 4, 8)
+    assert lib.aoh_cache_bytes(ctypes.byref(cfg), (ctypes.c_uint8 * 2)(0, 2)) == 0
+    assert "neither" in lib.aoh_last_error().decode()
+
+
+def test_init_rejects_null_and_small_buffers_before_any_cuda_call(lib):
+    cfg = aoh.make_config(1, 8, 2, 64, 64, 4, 8)
+    labels = (ctypes.c_uint8 * 2)(0, 1)
+    h = ctypes.c_void_p()
+    assert lib.aoh_cache_init(ctypes.byref(cfg), labels, None, 1 << 20, ctypes.byref(h)) == 1
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: the size check fails first
+    assert lib.aoh_cache_init(ctypes.byref(cfg), labels, fake, 16, ctypes.byref(h)) == 2
+    misaligned = ctypes.c_void_p((1 << 20) + 16)
+    assert lib.aoh_cache_init(ctypes.byref(cfg), labels, misaligned, 1 << 30, ctypes.byref(h)) == 1
+    unsupported = aoh.make_config(1, 12, 2, 64, 64, 4, 8)  # group of 6 is not compiled
+    assert lib.aoh_cache_init(ctypes.byref(unsupported), labels, fake, 1 << 30, ctypes.byref(h)) == 5
+
+
+def test_null_handle_calls_fail_cleanly(lib):
+    assert lib.aoh_prefill(None, None, None, 1, None, None, None, None) == 1
+    assert lib.aoh_decode_step(None, None, None, None, None, None) == 1
+    assert lib.aoh_cache_check(None, None) == 1
+    lib.aoh_cache_destroy(None)
