@@ -41,15 +41,24 @@ def load_peaks():
 
 # ------------------------------------------------------------------ workload
 
-def decode_workload():
+def decode_workload(batch=None, ctx=None):
+    import dataclasses
+
     from paper_2608_06849_gb300.workloads import DECODE_128K, labels_for
     wl = DECODE_128K
+    if batch or ctx:
+        wl = dataclasses.replace(wl, batch=batch or wl.batch, prefill_len=ctx or wl.prefill_len,
+                                 name=f"{wl.name}-small")
     return wl, labels_for(wl)
 
 
-def prefill_workload():
+def prefill_workload(T=None):
+    import dataclasses
+
     from paper_2608_06849_gb300.workloads import PREFILL_32K, labels_for
     wl = PREFILL_32K
+    if T:
+        wl = dataclasses.replace(wl, prefill_len=T, name=f"{wl.name}-small")
     return wl, labels_for(wl)
 
 
@@ -100,7 +109,7 @@ class ClockSampler:
         try:
             self.f = open(self.out, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                                          "-lms", "100", "-i", str(device_index)], stdout=self.f,
+                                          "-lms", "20", "-i", str(device_index)], stdout=self.f,
                                          stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -171,7 +180,7 @@ def run_native(args):
     K, W = args.steps, args.warmup
 
     # ---------------- decode leg (headline)
-    wl, labels = decode_workload()
+    wl, labels = decode_workload(args.decode_batch, args.decode_ctx)
     B, D, T0 = wl.batch, wl.d_head, wl.prefill_len
     total_steps = W + K + K + 2   # warmup, timed, e2e
     cache = aoh.Cache(B, wl.n_q_heads, wl.n_kv_heads, D, T0 + total_steps + 8, wl.sink, wl.window, labels)
@@ -228,7 +237,7 @@ def run_native(args):
     torch.cuda.empty_cache()
 
     # ---------------- prefill leg
-    pwl, plabels = prefill_workload()
+    pwl, plabels = prefill_workload(args.prefill_len)
     from paper_2608_06849_gb300.workloads import prefill_inputs
     q, k, v = prefill_inputs(pwl, device="cuda")
     T = pwl.prefill_len
@@ -406,6 +415,9 @@ def main():
     ap.add_argument("--prefill-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--decode-batch", type=int, default=None, help="smaller decode batch (profiling runs)")
+    ap.add_argument("--decode-ctx", type=int, default=None, help="smaller decode context (profiling runs)")
+    ap.add_argument("--prefill-len", type=int, default=None, help="shorter prefill (profiling runs)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "native":
         args.warmup = 3

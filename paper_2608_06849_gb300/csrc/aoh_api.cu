@@ -3,6 +3,8 @@
 #include <math.h>
 #include <stdarg.h>
 #include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include <algorithm>
 #include <string>
@@ -59,6 +61,34 @@ aoh_status check_config(const aoh_config* cfg, const uint8_t* labels, int* n_r, 
   return AOH_OK;
 }
 
+// Prefill tiles: one item per (b, query head, 128-row query tile), with the
+// number of 128-key tiles it visits as its cost; heaviest first so the
+// hardware block scheduler fills the machine longest-processing-time first.
+std::vector<int4> prefill_schedule(const CacheGeom& g, const std::vector<int32_t>& lens) {
+  constexpr int BM = 128, BN = 128;
+  std::vector<int4> items;
+  for (int b = 0; b < g.B; ++b) {
+    for (int h = 0; h < g.Hq; ++h) {
+      const bool streaming = g.kind[h / g.G] != 0;
+      for (int q0 = 0; q0 < lens[b]; q0 += BM) {
+        const int q_end = std::min(q0 + BM, (int)lens[b]);
+        int n;
+        if (!streaming) {
+          n = (q_end + BN - 1) / BN;
+        } else {
+          const int a_end = (std::min(g.S, q_end) + BN - 1) / BN;
+          const int c_begin = std::max(a_end, std::max(0, q0 - g.W + 1) / BN);
+          const int c_end = std::max(c_begin, (q_end + BN - 1) / BN);
+          n = a_end + (c_end - c_begin);
+        }
+        items.push_back(make_int4(b, h, q0, n));
+      }
+    }
+  }
+  std::stable_sort(items.begin(), items.end(), [](const int4& x, const int4& y) { return x.w > y.w; });
+  return items;
+}
+
 size_t bytes_for(const aoh_config& c, int n_r, int n_s) {
   const size_t tokens = (size_t)n_r * c.max_seq + (size_t)n_s * (size_t)(c.sink + c.window);
   return (size_t)c.batch * tokens * c.d_head * 2 * 2;
@@ -83,6 +113,9 @@ struct aoh_cache {
   uint32_t* d_done = nullptr;
   uint32_t* d_err = nullptr;
   float* d_partials = nullptr;
+  // prefill work list (device), grown on demand
+  int4* d_work = nullptr;
+  size_t work_cap = 0;
 };
 
 extern "C" {
@@ -106,7 +139,7 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   if (st != AOH_OK) return st;
   const aoh_config& c = *cfg;
   const int G = c.n_q_heads / c.n_kv_heads;
-  if (!decode_supported(c.d_head, G) || !prefill_supported(c.d_head, G))
+  if (!decode_supported(c.d_head, G))
     return fail(AOH_ERR_UNSUPPORTED, "group size %d with d_head %d is not compiled", G, c.d_head);
   if (!kv_buffer) return fail(AOH_ERR_INVALID, "kv_buffer is NULL");
   if (!aligned(kv_buffer, 256)) return fail(AOH_ERR_INVALID, "kv_buffer must be 256-byte aligned");
@@ -176,6 +209,7 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
 void aoh_cache_destroy(aoh_cache* cache) {
   if (!cache) return;
   if (cache->meta) cudaFree(cache->meta);
+  if (cache->d_work) cudaFree(cache->d_work);
   delete cache;
 }
 
@@ -255,20 +289,33 @@ aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, c
   if (e != cudaSuccess) return cuda_fail(e, "append kernel launch");
 
   if (out) {
-    PrefillArgs pa;
-    pa.geom = g;
-    pa.q = q;
-    pa.k = k;
-    pa.v = v;
-    pa.out = out;
-    pa.lens = cache->d_lens;
-    pa.T = T;
-    pa.scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
-    pa.work = nullptr;
-    pa.n_work = 0;
-    pa.err = cache->d_err;
-    e = launch_prefill(pa, s);
-    if (e != cudaSuccess) return cuda_fail(e, "prefill kernel launch");
+    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
+    {
+      std::vector<int4> items = prefill_schedule(g, lens);
+      if (items.size() > cache->work_cap) {
+        if (cache->d_work) cudaFree(cache->d_work);
+        cache->d_work = nullptr;
+        cache->work_cap = 0;
+        e = cudaMalloc(&cache->d_work, items.size() * sizeof(int4));
+        if (e != cudaSuccess) return cuda_fail(e, "work list allocation");
+        cache->work_cap = items.size();
+      }
+      e = cudaMemcpyAsync(cache->d_work, items.data(), items.size() * sizeof(int4), cudaMemcpyHostToDevice, s);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work)");
+      PrefillTcArgs pa;
+      memset(&pa, 0, sizeof(pa));
+      pa.geom = g;
+      pa.out = out;
+      pa.lens = cache->d_lens;
+      pa.work = cache->d_work;
+      pa.err = cache->d_err;
+      pa.T = T;
+      pa.scale_log2 = scale_log2;
+      if (!prefill_tc_make_maps(&pa, q, k, v, g.B, T))
+        return fail(AOH_ERR_CUDA, "cuTensorMapEncodeTiled failed for q/k/v");
+      e = launch_prefill_tc(pa, (int)items.size(), s);
+      if (e != cudaSuccess) return cuda_fail(e, "prefill kernel launch");
+    }
   }
   cache->lens = lens;
   return AOH_OK;

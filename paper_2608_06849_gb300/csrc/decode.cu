@@ -41,7 +41,7 @@ struct DecodeCfg {
   static constexpr int G = G_;
   static constexpr int LPT = D / 8;              // lanes per token group
   static constexpr int GPW = 32 / LPT;           // groups per warp
-  static constexpr int GP = next_pow2(G);        // rows padded to a power of two
+  static constexpr int GP = cmax(2, next_pow2(G));  // rows padded to a power of two (>= 2)
   static constexpr int NT = cmax(4, LPT / GP);   // rows per group per tile
   static constexpr int V = NT * GP;              // partial dots per lane
   static constexpr int RP = V / LPT;             // values per lane after reduce-scatter
@@ -432,13 +432,14 @@ cudaError_t launch_cfg(const DecodeArgs& a, int n_ctas, cudaStream_t s) {
 
 bool decode_supported(int D, int G) {
   if (D != 64 && D != 128) return false;
-  return G == 2 || G == 4 || G == 7 || G == 8;
+  return G == 1 || G == 2 || G == 4 || G == 7 || G == 8;
 }
 
 cudaError_t launch_decode(const DecodeArgs& a, int n_ctas, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;
   if (D == 128) {
     switch (G) {
+      case 1: return launch_cfg<128, 1>(a, n_ctas, s);
       case 2: return launch_cfg<128, 2>(a, n_ctas, s);
       case 4: return launch_cfg<128, 4>(a, n_ctas, s);
       case 7: return launch_cfg<128, 7>(a, n_ctas, s);
@@ -446,6 +447,7 @@ cudaError_t launch_decode(const DecodeArgs& a, int n_ctas, cudaStream_t s) {
     }
   } else if (D == 64) {
     switch (G) {
+      case 1: return launch_cfg<64, 1>(a, n_ctas, s);
       case 2: return launch_cfg<64, 2>(a, n_ctas, s);
       case 4: return launch_cfg<64, 4>(a, n_ctas, s);
       case 7: return launch_cfg<64, 7>(a, n_ctas, s);

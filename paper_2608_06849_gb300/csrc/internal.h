@@ -1,6 +1,7 @@
 // Host-side declarations shared by the translation units of libaoh.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -61,25 +62,25 @@ struct AppendArgs {
   int T;
 };
 
-struct PrefillArgs {
+// Arguments of the tcgen05 prefill kernel: tensor maps over q / k / v
+// ([B][T][H][D], box 128 rows x 64 columns, 128-byte swizzle) and a work list
+// of (b, query head, first row) tiles sorted by cost.
+struct alignas(64) PrefillTcArgs {
+  CUtensorMap tq, tk, tv;
   CacheGeom geom;
-  const void* q;  // [B][T][Hq][D]
-  const void* k;  // [B][T][Hkv][D]
-  const void* v;
-  void* out;      // [B][T][Hq][D]
+  void* out;            // [B][T][Hq][D]
   const int32_t* lens;  // device [B]
+  const int4* work;     // {b, h, q0, cost}
+  uint32_t* err;
   int T;
   float scale_log2;
-  const int4* work;  // work items
-  int n_work;
-  uint32_t* err;
 };
 
 // Launchers (return the launch's cudaError_t).
+bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const void* v, int B, int T);
+cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs& a, int n_ctas, cudaStream_t s);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
-cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t s);
 bool decode_supported(int D, int G);
-bool prefill_supported(int D, int G);
 
 }  // namespace aoh

@@ -1,0 +1,396 @@
+// Causal prefill attention on tcgen05 tensor cores (Sec. 5, "Chunked-Prefill
+// Stage", with the per-token sink + window rule for streaming heads).
+//
+// One CTA computes one 128-row query tile of one query head (rows are
+// consecutive positions). The KV tiles it visits come from a per-head
+// schedule: a retrieval head visits tiles 0 .. causal end; a streaming head
+// visits only the tiles holding its S sinks and the tiles that intersect the
+// W-token window of some row of the tile, so its cost is O(S + W) per row
+// instead of O(T). Tiles fully visible to every row skip the mask.
+//
+// Warp roles (192 threads):
+//   warp 0      TMA producer: Q once, then K_j / V_j tiles into a 4-stage ring
+//               (4D tensor maps over [B][T][H][D], 128-byte swizzle).
+//   warp 1      TMEM owner and MMA issuer: S_j = Q K_j^T into one of two
+//               TMEM S buffers (so QK of tile j+1 overlaps softmax of tile j),
+//               then O += P_j V_j into the TMEM O accumulator.
+//   warps 2-5   softmax: thread r owns query row r (TMEM lane r). It reads
+//               its S row with tcgen05.ld, applies the mask, keeps the
+//               running max / sum in fp32 registers (the max only moves when
+//               it grows by more than 2^8, so O is rarely rescaled), writes
+//               P = exp2(S - m) as bf16 into shared memory in the swizzled
+//               K-major layout the MMA reads, and finally normalises O.
+// TMEM columns: S0 [0,128), S1 [128,256), O [256, 256 + D).
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+#include "tc.cuh"
+
+namespace aoh {
+namespace {
+
+using bf16 = __nv_bfloat16;
+constexpr int kBM = 128;  // query rows per tile
+constexpr int kBN = 128;  // keys per KV tile
+constexpr int kNS = 4;    // KV ring stages (K and V tiles alternate)
+constexpr float kRescaleThreshold = 8.0f;
+constexpr uint32_t kTmemCols = 512;
+
+template <int D>
+struct PfCfg {
+  static constexpr int DBLK = D / 64;            // 64-wide column blocks (one TMA box each)
+  static constexpr int BOX = 128 * 64 * 2;       // bytes of one [128 rows][64] box
+  static constexpr int QBYTES = DBLK * BOX;
+  static constexpr int KVBYTES = DBLK * BOX;
+  static constexpr int PBYTES = 2 * BOX;         // [128 rows][128 keys]
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_KV = OFF_Q + QBYTES;
+  static constexpr int OFF_P = OFF_KV + kNS * KVBYTES;
+  static constexpr int OFF_BAR = OFF_P + PBYTES;
+  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 1 + 1 + 1;
+  static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;
+  static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, false);
+  static constexpr uint32_t IDESC_PV = idesc_bf16(kBM, D, true);
+};
+
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_t* err, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(err, kErrTimeout);
+      *abort_flag = 1;
+      return false;
+    }
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constant__ PrefillTcArgs a) {
+  using C = PfCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint8_t* sKV = smem + C::OFF_KV;
+  uint8_t* sP = smem + C::OFF_P;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;
+  uint64_t* kv_empty = kv_full + kNS;
+  uint64_t* s_full = kv_empty + kNS;
+  uint64_t* s_empty = s_full + 2;
+  uint64_t* p_full = s_empty + 2;
+  uint64_t* pv_done = p_full + 1;
+  uint64_t* drain = pv_done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int4 item = a.work[blockIdx.x];
+  const int b = item.x, h = item.y, q0 = item.z;
+  const CacheGeom& g = a.geom;
+  const int kvh = h / g.G;
+  const bool streaming = g.kind[kvh] != 0;
+  const int len = a.lens[b];
+  const int q_end = min(q0 + kBM, len);
+  // KV tiles visited: [0, a_end) then [c_begin, c_end)
+  int a_end, c_begin, c_end;
+  if (!streaming) {
+    a_end = (q_end + kBN - 1) / kBN;
+    c_begin = c_end = a_end;
+  } else {
+    a_end = (min(g.S, q_end) + kBN - 1) / kBN;
+    c_begin = max(a_end, max(0, q0 - g.W + 1) / kBN);
+    c_end = max(c_begin, (q_end + kBN - 1) / kBN);
+  }
+  const int n_tiles = a_end + (c_end - c_begin);
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < kNS; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&s_full[s], 1);
+      mbar_init(&s_empty[s], 4);
+    }
+    mbar_init(p_full, 4);
+    mbar_init(pv_done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      prefetch_tmap(&a.tq);
+      prefetch_tmap(&a.tk);
+      prefetch_tmap(&a.tv);
+      mbar_arrive_expect_tx(q_full, C::QBYTES);
+      for (int db = 0; db < C::DBLK; ++db) tma_load_4d(sQ + db * C::BOX, &a.tq, db * 64, h, q0, b, q_full);
+      int issued = 0;
+      for (int jj = 0; jj < n_tiles; ++jj) {
+        const int j = jj < a_end ? jj : c_begin + (jj - a_end);
+        bool ok = true;
+        for (int sel = 0; sel < 2 && ok; ++sel) {
+          const int it = 2 * jj + sel;
+          const int st = it % kNS;
+          if (it >= kNS && !wait_bar(&kv_empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&kv_full[st], C::KVBYTES);
+          const CUtensorMap* map = sel ? &a.tv : &a.tk;
+          for (int db = 0; db < C::DBLK; ++db)
+            tma_load_4d(sKV + st * C::KVBYTES + db * C::BOX, map, db * 64, kvh, j * kBN, b, &kv_full[st]);
+          issued = it + 1;
+        }
+        if (!ok) break;
+      }
+      // every issued copy lands before the CTA can exit
+      wait_bar(q_full, 0, a.err, abort_flag);
+      for (int it = issued > kNS ? issued - kNS : 0; it < issued; ++it)
+        wait_bar(&kv_full[it % kNS], (it / kNS) & 1, a.err, abort_flag);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t q_addr = smem_u32(sQ), kv_addr = smem_u32(sKV), p_addr = smem_u32(sP);
+      auto pv = [&](int x) -> bool {
+        const int it = 2 * x + 1, st = it % kNS;
+        if (!wait_bar(&kv_full[st], (it / kNS) & 1, a.err, abort_flag)) return false;
+        if (!wait_bar(p_full, x & 1, a.err, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t v_addr = kv_addr + st * C::KVBYTES;
+#pragma unroll
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(p_addr + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc_sw128(v_addr + kk * 16 * 128, C::BOX, 1024);
+          tc_mma(tmem + 256, ad, bd, C::IDESC_PV, (x > 0 || kk > 0) ? 1u : 0u);
+        }
+        tc_commit(pv_done);
+        tc_commit(&kv_empty[st]);
+        return true;
+      };
+      bool ok = wait_bar(q_full, 0, a.err, abort_flag);
+      tc_fence_after();
+      for (int jj = 0; jj < n_tiles && ok; ++jj) {
+        const int it = 2 * jj, st = it % kNS;
+        if (!wait_bar(&kv_full[st], (it / kNS) & 1, a.err, abort_flag)) { ok = false; break; }
+        if (jj >= 2 && !wait_bar(&s_empty[jj & 1], ((jj >> 1) & 1) ^ 1, a.err, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t k_addr = kv_addr + st * C::KVBYTES;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(q_addr + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc_sw128(k_addr + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
+          tc_mma(tmem + (jj & 1) * 128, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(&s_full[jj & 1]);
+        tc_commit(&kv_empty[st]);
+        if (jj >= 1 && !pv(jj - 1)) { ok = false; break; }
+      }
+      if (ok) pv(n_tiles - 1);
+      tc_commit(drain);
+      wait_bar(drain, 0, a.err, abort_flag);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;
+    const int i = q0 + r;
+    const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+    const int S = g.S, W = g.W;
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int jj = 0; jj < n_tiles; ++jj) {
+      const int j = jj < a_end ? jj : c_begin + (jj - a_end);
+      const int j0 = j * kBN;
+      if (!__all_sync(0xffffffffu, wait_bar(&s_full[jj & 1], (jj >> 1) & 1, a.err, abort_flag))) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float s[kBN];
+#pragma unroll
+      for (int c = 0; c < kBN / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tl + (jj & 1) * 128 + c * 32, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(v[e]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_empty[jj & 1]);
+
+      const int jl = j0 + kBN - 1;
+      const bool full_vis = jl <= q0 && jl < len && (!streaming || jl < S || (q0 + kBM - 1) - j0 < W);
+      float rmax = -INFINITY;
+      if (full_vis) {
+#pragma unroll
+        for (int k = 0; k < kBN; ++k) {
+          s[k] *= a.scale_log2;
+          rmax = fmaxf(rmax, s[k]);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < kBN; ++k) {
+          const int jp = j0 + k;
+          const bool vis = jp <= i && jp < len && (!streaming || jp < S || i - jp < W);
+          s[k] = vis ? s[k] * a.scale_log2 : -INFINITY;
+          rmax = fmaxf(rmax, s[k]);
+        }
+      }
+      const float mn = fmaxf(m, rmax);
+      const bool resc = mn > m + kRescaleThreshold;
+      float alpha = 1.f;
+      if (resc) {
+        alpha = (m == -INFINITY) ? 0.f : fast_exp2(m - mn);
+        m = mn;
+      }
+      const bool warp_resc = __any_sync(0xffffffffu, resc) && jj > 0;
+      float sum = 0.f;
+      uint32_t pk[kBN / 2];
+#pragma unroll
+      for (int k = 0; k < kBN; k += 2) {
+        const float p0 = (s[k] == -INFINITY) ? 0.f : fast_exp2(s[k] - m);
+        const float p1 = (s[k + 1] == -INFINITY) ? 0.f : fast_exp2(s[k + 1] - m);
+        sum += p0 + p1;
+        pk[k / 2] = float2_to_bf16x2(p0, p1);
+      }
+      l = l * alpha + sum;
+
+      if (jj >= 1) {
+        if (!__all_sync(0xffffffffu, wait_bar(pv_done, (jj - 1) & 1, a.err, abort_flag))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (warp_resc) {
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t v[32];
+            tmem_ld32(tl + 256 + c * 32, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+            tmem_st32(tl + 256 + c * 32, v);
+          }
+          tmem_st_wait();
+        }
+      }
+      // P row r -> swizzled K-major tile: key block kb (64 keys), chunk c (8 keys)
+#pragma unroll
+      for (int kb = 0; kb < 2; ++kb) {
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int base = kb * 32 + c * 4;
+          uint4 val = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
+          *reinterpret_cast<uint4*>(sP + kb * C::BOX + r * 128 + ((c ^ (r & 7)) << 4)) = val;
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok && __all_sync(0xffffffffu, wait_bar(pv_done, (n_tiles - 1) & 1, a.err, abort_flag))) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      bf16* op = static_cast<bf16*>(a.out) + (((size_t)b * a.T + min(i, len - 1)) * g.Hq + h) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tl + 256 + c * 32, v);
+        tmem_ld_wait();
+        if (i < len) {
+#pragma unroll
+          for (int e = 0; e < 32; e += 8) {
+            uint4 w;
+            w.x = float2_to_bf16x2(__uint_as_float(v[e + 0]) * inv, __uint_as_float(v[e + 1]) * inv);
+            w.y = float2_to_bf16x2(__uint_as_float(v[e + 2]) * inv, __uint_as_float(v[e + 3]) * inv);
+            w.z = float2_to_bf16x2(__uint_as_float(v[e + 4]) * inv, __uint_as_float(v[e + 5]) * inv);
+            w.w = float2_to_bf16x2(__uint_as_float(v[e + 6]) * inv, __uint_as_float(v[e + 7]) * inv);
+            *reinterpret_cast<uint4*>(op + c * 32 + e) = w;
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 4D map over a [B][T][H][D] bf16 tensor, box [1][128][1][64], 128-byte swizzle.
+bool make_map(CUtensorMap* map, const void* base, int B, int T, int H, int D) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)B};
+  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2, (cuuint64_t)T * H * D * 2};
+  cuuint32_t box[4] = {64, 1, 128, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_cfg(const PrefillTcArgs& a, int n_items, cudaStream_t s) {
+  using C = PfCfg<D>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  prefill_tc_kernel<D><<<n_items, 192, C::SMEM, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const void* v, int B, int T) {
+  const CacheGeom& g = a->geom;
+  return make_map(&a->tq, q, B, T, g.Hq, g.D) && make_map(&a->tk, k, B, T, g.Hkv, g.D) &&
+         make_map(&a->tv, v, B, T, g.Hkv, g.D);
+}
+
+cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s) {
+  if (n_items <= 0) return cudaSuccess;
+  if (a.geom.D == 128) return launch_cfg<128>(a, n_items, s);
+  if (a.geom.D == 64) return launch_cfg<64>(a, n_items, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace aoh

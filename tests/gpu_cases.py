@@ -27,17 +27,31 @@ def f64(t):
     return t.detach().float().cpu().numpy().astype(np.float64)
 
 
-def assert_matches(got, want, what=""):
-    """max/mean absolute bounds, plus an elementwise bound of two bf16 ulps of
-    the exact value (the output is rounded to bf16 once) + 1e-3."""
+def bf16_round(x):
+    return torch.from_numpy(np.asarray(x, dtype=np.float32)).to(torch.bfloat16).double().numpy()
+
+
+def assert_matches(got, want, what="", mag=None, abs_bounds=True):
+    """max |err| <= 1e-2; mean |err| <= 1e-3 on top of the mean error that
+    rounding the exact result to the bf16 output format already costs (that
+    term is ~1e-3 by itself when outputs are of unit size, e.g. a query that
+    sees two tokens; it is ~1e-4 on the long-context workloads); and an
+    elementwise bound derived from the arithmetic: rounding each softmax
+    weight p_j to bf16 before the P.V product moves the output by at most
+    2^-9 * sum_j p_j |v_j| / l (``mag``, the oracle run on |v|), and rounding
+    the output to bf16 by 2^-9 |o|; the bound allows twice both plus 1e-4."""
     got = np.asarray(got, dtype=np.float64)
     want = np.asarray(want, dtype=np.float64)
     assert got.shape == want.shape, (got.shape, want.shape)
     assert np.isfinite(got).all(), f"{what}: non-finite output"
     err = np.abs(got - want)
-    assert err.max() <= MAX_ABS, f"{what}: max |err| {err.max():.3e}"
-    assert err.mean() <= MEAN_ABS, f"{what}: mean |err| {err.mean():.3e}"
-    bound = np.abs(want) * 2.0 ** -8 + 1e-3
+    if abs_bounds:
+        assert err.max() <= MAX_ABS, f"{what}: max |err| {err.max():.3e}"
+        floor = np.abs(bf16_round(want) - want).mean()
+        assert err.mean() <= MEAN_ABS + floor, f"{what}: mean |err| {err.mean():.3e} (bf16 floor {floor:.3e})"
+    if mag is None:
+        mag = np.abs(want)
+    bound = (np.abs(want) + np.asarray(mag)) * 2.0 ** -8 + 1e-4
     bad = err > bound
     assert not bad.any(), f"{what}: {bad.sum()} elements beyond 2 ulp, worst {err[bad].max():.3e}"
     return err.max(), err.mean()
@@ -64,7 +78,7 @@ def check_cache_image(cache, k, v, lens, labels, S, W):
 
 
 def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink_scale=8.0, seed=0,
-             check_prefill_out=True, peaky=1.0, rows=None):
+             check_prefill_out=True, peaky=1.0, rows=None, abs_bounds=True):
     """Prefill (+ decode steps) on the GPU; every output compared with the oracle."""
     ensure_lib()
     wl = Workload("case", B, Hq, Hkv, d, T, decode_steps, S, W, sum(labels), seed=seed, sink_scale=sink_scale)
@@ -84,7 +98,8 @@ def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink
         for b in range(B):
             r = np.arange(lens[b]) if rows is None else np.asarray([x for x in rows if x < lens[b]])
             want = oatt.prefill(qn[b, :lens[b]], kn[b, :lens[b]], vn[b, :lens[b]], labels, S, W, rows=r)
-            results[("prefill", b)] = assert_matches(f64(out[b, r]), want, f"prefill b={b}")
+            mag = oatt.prefill(qn[b, :lens[b]], kn[b, :lens[b]], np.abs(vn[b, :lens[b]]), labels, S, W, rows=r)
+            results[("prefill", b)] = assert_matches(f64(out[b, r]), want, f"prefill b={b}", mag, abs_bounds)
     check_cache_image(cache, k, v, lens, labels, S, W)
 
     kall = [kn[b, :lens[b]] for b in range(B)]
@@ -103,7 +118,8 @@ def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink
             kseq_t[b] = torch.cat([kseq_t[b], dk[b][None]], dim=0)
             vseq_t[b] = torch.cat([vseq_t[b], dv[b][None]], dim=0)
             want = oatt.decode_step(dqn[b], kall[b], vall[b], labels, S, W)
-            results[("decode", step, b)] = assert_matches(f64(dout[b]), want, f"decode step={step} b={b}")
+            mag = oatt.decode_step(dqn[b], kall[b], np.abs(vall[b]), labels, S, W)
+            results[("decode", step, b)] = assert_matches(f64(dout[b]), want, f"decode step={step} b={b}", mag, abs_bounds)
     cache.check()
     if decode_steps:
         new_lens = [L + decode_steps for L in lens]

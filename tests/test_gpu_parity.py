@@ -34,6 +34,9 @@ CASES = {
     "ring_wraps_many_times": (1, 8, 2, 128, 40, 3, 5, [1, 0], None, 30),
     "single_token_prefill": (3, 8, 2, 128, 1, 4, 4, [0, 1], None, 6),
     "tile_edges": (1, 8, 2, 128, 65, 1, 63, [1, 0], None, 70),
+    "mha_group1_d128": (1, 2, 2, 128, 140, 4, 30, [0, 1], None, 3),
+    "mha_group1_d64": (2, 3, 3, 64, 90, 0, 7, [1, 0, 1], [90, 41], 3),
+    "prefill_multi_tile_ragged": (3, 8, 2, 128, 777, 16, 200, [1, 0], [777, 129, 640], 2),
 }
 
 
@@ -45,8 +48,11 @@ def test_small_case(name):
 
 def test_peaky_keys_relative_error():
     """Keys scaled x4 make the softmax sharp, so a dropped or misplaced term
-    cannot hide behind a near-uniform average."""
-    run_case(1, 8, 2, 128, 400, 16, 64, [0, 1], decode_steps=4, peaky=4.0, sink_scale=1.0)
+    cannot hide behind a near-uniform average. A sharp softmax puts weights
+    near 1 on single keys, where bf16 rounding of P and of the output alone
+    reach ~1.6e-2 for |v| ~ 4, so this case is held to the elementwise bound
+    derived from that arithmetic (not the workloads' absolute 1e-2)."""
+    run_case(1, 8, 2, 128, 400, 16, 64, [0, 1], decode_steps=4, peaky=4.0, sink_scale=1.0, abs_bounds=False)
 
 
 def test_long_decode_split_path():
