@@ -321,8 +321,8 @@ def traffic_for(kernel):
         d = json.load(open(p)).get(kernel)
         if not d:
             return None
-        from paper_2608_06849_gb300.build import source_digest
-        if d.get("source_digest") != source_digest():
+        from paper_2608_06849_gb300.build import kernel_digest
+        if d.get("kernel_digest") != kernel_digest(kernel):
             return None
         return d.get("bytes_per_launch")
     except Exception:

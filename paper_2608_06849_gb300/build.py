@@ -33,6 +33,23 @@ def source_digest():
     return h.hexdigest()[:16]
 
 
+KERNEL_SOURCES = {
+    "decode": ["decode.cu", "common.cuh"],
+    "prefill": ["prefill_tc.cu", "tc.cuh", "common.cuh"],
+}
+
+
+def kernel_digest(kernel):
+    """sha256 over one kernel's own device sources (identifies that kernel's code)."""
+    import hashlib
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES[kernel]:
+        f = os.path.join(CSRC, name)
+        h.update(name.encode())
+        h.update(open(f, "rb").read())
+    return h.hexdigest()[:16]
+
+
 def _compile(src, verbose):
     obj = os.path.join(OBJ, os.path.basename(src)[:-3] + ".o")
     cmd = [NVCC, *ARCH, *FLAGS, "-c", src, "-o", obj]
