@@ -162,6 +162,53 @@ void aoh_cache_destroy(aoh_cache* cache);
 /* Message of the last failed call on this thread ("" if none). */
 const char* aoh_last_error(void);
 
+/*
+ * A decode step for callers that cannot allocate device memory (the paper has
+ * no counterpart; this is a deployment convenience of the library).
+ *
+ * Who needs it: a caller that must not allocate device memory once it is
+ * running, e.g. an inference server that reserves its whole memory arena at
+ * start-up and treats any later cudaMalloc as an error, or a latency-critical
+ * loop that cannot absorb cudaMalloc's implicit device-wide synchronisation.
+ * aoh_cache_init allocates a small metadata block, so such callers cannot use
+ * the handle API for decode. This call runs the same split-KV decode kernel
+ * as aoh_decode_step with no handle and performs no device allocation: its
+ * scratch (split partials, arrival counters, an error word) lives in one
+ * statically allocated device array of 16 MiB + 64 KiB inside the library,
+ * which every GPU that loads the library holds until the process exits.
+ *
+ *   cfg, head_labels  as for aoh_cache_init (host memory, not retained).
+ *   kv_buffer  the KV cache in the layout aoh_cache_init documents (e.g.
+ *              filled by aoh_prefill through a handle, or written by the
+ *              caller); 256-byte aligned. The new token's K/V is appended.
+ *   lens       device int32 [B]: tokens held per sequence before the step;
+ *              each entry is advanced by one on the device.
+ *   max_len    host upper bound of every lens[b]; used for the split schedule
+ *              and the capacity check (max_len + 1 <= max_seq when a
+ *              retrieval head exists).
+ *   q, k_new, v_new, out  as for aoh_decode_step.
+ *
+ * Limits and behaviour:
+ *   - batch * n_kv_heads must be <= 16320 (AOH_ERR_CAPACITY otherwise). When
+ *     the partial space is too small for the usual split count, fewer splits
+ *     are used.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current) and caches it; make
+ *     that first call before any stream capture.
+ *   - Every call shares the one array and leaves its contents behind; the
+ *     counters that must start at zero are cleared on the stream at the start
+ *     of each call. Calls whose kernels overlap on the GPU (on different
+ *     streams, or from different threads without ordering) race on the
+ *     scratch and produce wrong results: order them on one stream.
+ *   - A bounded-wait timeout inside the kernel is recorded only in the
+ *     scratch error word, which this call does not report; the outputs of
+ *     such a call are unspecified.
+ * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
+ */
+aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
+                                   int32_t* lens, int32_t max_len, const void* q, const void* k_new,
+                                   const void* v_new, void* out, void* stream);
+
 /* Library ABI version (major * 100 + minor). */
 int32_t aoh_version(void);
 

@@ -34,6 +34,7 @@ EXPORTS = [
     "aoh_cache_destroy",
     "aoh_last_error",
     "aoh_version",
+    "aoh_decode_step_noalloc",
 ]
 
 
@@ -77,6 +78,7 @@ def load():
         "aoh_cache_destroy": (None, [P]),
         "aoh_last_error": (ctypes.c_char_p, []),
         "aoh_version": (i32, []),
+        "aoh_decode_step_noalloc": (i32, [cfgp, u8p, P, i32p, i32, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -143,6 +145,17 @@ def aoh_prefill(q, k, v, T, seq_lens, cache, out, stream=None):
 def aoh_decode_step(q, k_new, v_new, cache, out, stream=None):
     _check(load().aoh_decode_step(_ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), cache,
                                   _ptr(out, "out"), _stream_ptr(stream)))
+
+
+def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream=None):
+    """The allocation-free decode step: ``kv_buffer`` (CUDA uint8) and ``lens``
+    (CUDA int32 [B], advanced by one on the device) belong to the caller."""
+    if not lens.is_cuda or lens.dtype != torch.int32 or not lens.is_contiguous():
+        raise ValueError("lens must be a contiguous int32 CUDA tensor")
+    _check(load().aoh_decode_step_noalloc(
+        ctypes.byref(cfg), _labels_arr(labels), _ptr(kv_buffer, "kv_buffer", torch.uint8),
+        ctypes.cast(ctypes.c_void_p(lens.data_ptr()), ctypes.POINTER(ctypes.c_int32)), int(max_len),
+        _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), _ptr(out, "out"), _stream_ptr(stream)))
 
 
 def aoh_cache_lens(cache, batch):

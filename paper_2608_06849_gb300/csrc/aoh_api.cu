@@ -96,6 +96,8 @@ size_t bytes_for(const aoh_config& c, int n_r, int n_s) {
 
 }  // namespace
 
+void aoh::record_error(const char* msg) { g_last_error = msg; }
+
 struct aoh_cache {
   aoh_config cfg;
   CacheGeom geom;

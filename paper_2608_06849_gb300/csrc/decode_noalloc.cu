@@ -1,0 +1,163 @@
+// A decode step for callers that cannot allocate device memory.
+//
+// Some callers must not allocate device memory once they are running: an
+// inference server that reserves its whole memory arena at start-up and
+// treats any later cudaMalloc as a failure, or a latency-critical loop where
+// cudaMalloc's implicit device-wide synchronisation would stall every other
+// stream. aoh_cache_init allocates a small metadata block, so those callers
+// cannot use the handle API for decode. This entry point runs the same
+// split-KV decode kernel, but its scratch (split partials, arrival counters,
+// the error word) lives in one statically allocated device array of this
+// file, sized kNoAllocScratchBytes. Every GPU that loads the library holds
+// that array until the process exits.
+//
+// The array's host-side name is only a stand-in for the device symbol, so the
+// device address is looked up with cudaGetSymbolAddress the first time a
+// device calls in (with that device current) and cached per device.
+#include <math.h>
+#include <stdio.h>
+
+#include <mutex>
+
+#include "../../include/aoh.h"
+#include "internal.h"
+
+namespace aoh {
+namespace {
+
+constexpr size_t kNoAllocHeaderBytes = 64 * 1024;         // err, done, per-(b, head) counters
+constexpr size_t kNoAllocPartialBytes = 16u * 1024 * 1024;  // split-KV partials
+constexpr size_t kNoAllocScratchBytes = kNoAllocHeaderBytes + kNoAllocPartialBytes;
+constexpr int kNoAllocMaxItems = (int)(kNoAllocHeaderBytes / 4) - 64;  // B * n_kv_heads limit
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_setup_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+int g_num_sms[kMaxDevices] = {};
+
+aoh_status set_err(aoh_status st, const char* msg) {
+  record_error(msg);
+  return st;
+}
+
+}  // namespace
+}  // namespace aoh
+
+using namespace aoh;
+
+extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
+                                              int32_t* lens, int32_t max_len, const void* q, const void* k_new,
+                                              const void* v_new, void* out, void* stream) {
+  if (!cfg || !head_labels || !kv_buffer || !lens || !q || !k_new || !v_new || !out)
+    return set_err(AOH_ERR_INVALID, "aoh_decode_step_noalloc: NULL argument");
+  const aoh_config& c = *cfg;
+  if (c.batch < 1 || c.n_q_heads < 1 || c.n_kv_heads < 1 || c.n_kv_heads > kMaxKvHeads || c.max_seq < 1 ||
+      c.n_q_heads % c.n_kv_heads || (c.d_head != 64 && c.d_head != 128) || c.sink < 0 || c.window < 1)
+    return set_err(AOH_ERR_INVALID, "aoh_decode_step_noalloc: invalid config");
+  const int G = c.n_q_heads / c.n_kv_heads;
+  if (!decode_supported(c.d_head, G))
+    return set_err(AOH_ERR_UNSUPPORTED, "aoh_decode_step_noalloc: group size not compiled");
+  const uintptr_t al = reinterpret_cast<uintptr_t>(kv_buffer) | reinterpret_cast<uintptr_t>(q) |
+                       reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new) |
+                       reinterpret_cast<uintptr_t>(out);
+  if (al % 16 || reinterpret_cast<uintptr_t>(kv_buffer) % 256)
+    return set_err(AOH_ERR_INVALID, "aoh_decode_step_noalloc: misaligned pointer");
+  const int items = c.batch * c.n_kv_heads;
+  if (items > kNoAllocMaxItems)
+    return set_err(AOH_ERR_CAPACITY,
+                   "aoh_decode_step_noalloc: batch * n_kv_heads exceeds the static scratch limit of 16320");
+
+  CacheGeom g;
+  g.B = c.batch;
+  g.Hq = c.n_q_heads;
+  g.Hkv = c.n_kv_heads;
+  g.D = c.d_head;
+  g.G = G;
+  g.max_seq = c.max_seq;
+  g.S = c.sink;
+  g.W = c.window;
+  int n_r = 0, n_s = 0;
+  for (int h = 0; h < c.n_kv_heads; ++h) {
+    if (head_labels[h] == AOH_RETRIEVAL) {
+      g.kind[h] = 0;
+      g.idx[h] = (uint8_t)n_r;
+      g.r_head[n_r++] = (uint8_t)h;
+    } else if (head_labels[h] == AOH_STREAMING) {
+      g.kind[h] = 1;
+      g.idx[h] = (uint8_t)n_s;
+      g.s_head[n_s++] = (uint8_t)h;
+    } else {
+      return set_err(AOH_ERR_INVALID, "aoh_decode_step_noalloc: bad head label");
+    }
+  }
+  g.n_r = n_r;
+  g.n_s = n_s;
+  if (max_len < 0) return set_err(AOH_ERR_INVALID, "aoh_decode_step_noalloc: max_len < 0");
+  if (n_r > 0 && max_len + 1 > c.max_seq)
+    return set_err(AOH_ERR_CAPACITY, "aoh_decode_step_noalloc: a retrieval head would pass max_seq");
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+    return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaGetDevice failed");
+  void* scratch = nullptr;
+  int num_sms = 0;
+  {
+    std::lock_guard<std::mutex> lock(g_setup_mutex);
+    if (!g_scratch_ptr[dev]) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+      if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaGetSymbolAddress failed");
+      int sms = 0;
+      e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: device query failed");
+      g_num_sms[dev] = sms;
+      g_scratch_ptr[dev] = p;
+    }
+    scratch = g_scratch_ptr[dev];
+    num_sms = g_num_sms[dev];
+  }
+  uint32_t* header = static_cast<uint32_t*>(scratch);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // err, done and the arrival counters must start at zero; clear them every call.
+  e = cudaMemsetAsync(header, 0, (size_t)(64 + items) * 4, s);
+  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaMemsetAsync failed");
+
+  // Split schedule as the handle API computes it, bounded by the partial space.
+  const size_t per_split = (size_t)items * G * (c.d_head + 2) * 4;
+  int stride = (int)(kNoAllocPartialBytes / per_split);
+  if (stride > kMaxSplits) stride = kMaxSplits;
+  if (stride < 1) stride = 1;
+  const int maxlen = max_len + 1;
+  const int win = maxlen < c.sink + c.window ? maxlen : c.sink + c.window;
+  const double total = (double)c.batch * ((double)n_r * maxlen + (double)n_s * win);
+  const double target = (double)num_sms * 2 * 4;
+  int chunk = (int)(total / target + 0.999999);
+  if (chunk < 512) chunk = 512;
+  int ns_r = n_r ? (maxlen + chunk - 1) / chunk : 0;
+  int ns_s = n_s ? (win + chunk - 1) / chunk : 0;
+  if (n_r) ns_r = ns_r < 1 ? 1 : (ns_r > stride ? stride : ns_r);
+  if (n_s) ns_s = ns_s < 1 ? 1 : (ns_s > stride ? stride : ns_s);
+
+  DecodeArgs a;
+  a.geom = g;
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.out = out;
+  a.kv = kv_buffer;
+  a.lens = lens;
+  a.err = header;
+  a.done = header + 32;
+  a.counters = header + 64;
+  a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
+  a.ns_r = ns_r;
+  a.ns_s = ns_s;
+  a.split_stride = stride;
+  a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));
+  e = launch_decode(a, c.batch * (n_r * ns_r + n_s * ns_s), s);
+  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: kernel launch failed");
+  return AOH_OK;
+}

@@ -76,6 +76,9 @@ struct alignas(64) PrefillTcArgs {
   float scale_log2;
 };
 
+// Store `msg` as the calling thread's aoh_last_error() message.
+void record_error(const char* msg);
+
 // Launchers (return the launch's cudaError_t).
 bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const void* v, int B, int T);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);

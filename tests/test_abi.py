@@ -42,6 +42,18 @@ def test_every_declared_symbol_is_exported(lib):
     assert sorted(aoh.EXPORTS) == declared_functions()
 
 
+def test_noalloc_rejects_bad_arguments_on_host(lib):
+    cfg = aoh.make_config(1, 8, 2, 64, 64, 4, 8)
+    labels = (ctypes.c_uint8 * 2)(0, 1)
+    fake = ctypes.c_void_p(1 << 20)
+    assert lib.aoh_decode_step_noalloc(ctypes.byref(cfg), labels, None, None, 0, fake, fake, fake, fake, None) == 1
+    big = aoh.make_config(4096, 8, 8, 64, 64, 4, 8)  # 32768 (b, head) items > 16320
+    labels8 = (ctypes.c_uint8 * 8)(*([0] * 8))
+    lens = ctypes.cast(fake, ctypes.POINTER(ctypes.c_int32))
+    assert lib.aoh_decode_step_noalloc(ctypes.byref(big), labels8, fake, lens, 0, fake, fake, fake, fake, None) == 2
+    assert "16320" in lib.aoh_last_error().decode()
+
+
 def test_version(lib):
     assert aoh.aoh_version() == 100
 
