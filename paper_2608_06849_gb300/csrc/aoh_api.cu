@@ -107,7 +107,6 @@ struct aoh_cache {
   std::vector<int32_t> lens;  // host mirror of the device lengths
   int device = 0;
   int num_sms = 0;
-  int split_stride = 1;
   // device metadata (one allocation)
   void* meta = nullptr;
   int32_t* d_lens = nullptr;
@@ -184,11 +183,9 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
     delete h;
     return cuda_fail(e, "cudaGetDevice");
   }
-  const int longest = std::max(c.max_seq, c.sink + c.window);
-  h->split_stride = std::min(kMaxSplits, std::max(1, (longest + 511) / 512));
   const size_t n_lens = ((size_t)c.batch + 63) / 64 * 64;
   const size_t n_cnt = ((size_t)c.batch * c.n_kv_heads + 63) / 64 * 64;
-  const size_t n_part = (size_t)c.batch * c.n_kv_heads * h->split_stride * G * (c.d_head + 2);
+  const size_t n_part = decode_partial_floats(2 * h->num_sms, G, c.d_head);
   const size_t meta_bytes = (n_lens + n_cnt + 64) * 4 + n_part * 4;
   e = cudaMalloc(&h->meta, meta_bytes);
   if (e == cudaSuccess) e = cudaMemset(h->meta, 0, meta_bytes);
@@ -330,23 +327,13 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
   if (!aligned(q, 16) || !aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(out, 16))
     return fail(AOH_ERR_INVALID, "q, k_new, v_new and out must be 16-byte aligned");
   const CacheGeom& g = cache->geom;
-  int maxlen = 0;
+  long long total = 0;
   for (int b = 0; b < g.B; ++b) {
     if (g.n_r > 0 && cache->lens[b] + 1 > g.max_seq)
       return fail(AOH_ERR_CAPACITY, "sequence %d holds %d tokens; max_seq is %d", b, cache->lens[b], g.max_seq);
-    maxlen = std::max(maxlen, cache->lens[b] + 1);
+    const long long t1 = cache->lens[b] + 1;
+    total += g.n_r * t1 + g.n_s * std::min<long long>(t1, g.S + g.W);
   }
-  // Split-KV schedule: rows per split chosen so the launch holds a few waves
-  // of CTAs; streaming heads get splits of about the same size.
-  const int win = std::min(maxlen, g.S + g.W);
-  double total = 0;
-  for (int b = 0; b < g.B; ++b)
-    total += (double)g.n_r * (cache->lens[b] + 1) + (double)g.n_s * std::min(cache->lens[b] + 1, g.S + g.W);
-  const double target_ctas = (double)cache->num_sms * 2 * 4;
-  const int chunk = std::max(512, (int)ceil(total / target_ctas));
-  const int ns_r = g.n_r ? std::min(cache->split_stride, std::max(1, (maxlen + chunk - 1) / chunk)) : 0;
-  const int ns_s = g.n_s ? std::min(cache->split_stride, std::max(1, (win + chunk - 1) / chunk)) : 0;
-
   DecodeArgs a;
   a.geom = g;
   a.q = q;
@@ -359,12 +346,9 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
   a.counters = cache->d_counters;
   a.done = cache->d_done;
   a.err = cache->d_err;
-  a.ns_r = ns_r;
-  a.ns_s = ns_s;
-  a.split_stride = cache->split_stride;
+  a.n_ctas = decode_ctas(total, cache->num_sms);
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
-  const int n_ctas = g.B * (g.n_r * ns_r + g.n_s * ns_s);
-  cudaError_t e = launch_decode(a, n_ctas, (cudaStream_t)stream);
+  cudaError_t e = launch_decode(a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");
   for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
   return AOH_OK;

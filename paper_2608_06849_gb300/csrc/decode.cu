@@ -50,15 +50,16 @@ struct DecodeCfg {
   static constexpr int NG = NW * GPW;            // groups per CTA
   static constexpr int TOK = NG * NT;            // rows per tile
   static constexpr int RB = D * 2;               // bytes per row
-  static constexpr int NST = 6;                  // pipeline stages
+  static constexpr int NST = G <= 4 ? 6 : 5;    // pipeline stages
   static constexpr int STAGE_BYTES = TOK * RB * 2;
   static constexpr int DATA_BYTES = NST * STAGE_BYTES;
-  static constexpr int MERGE_BYTES = NG * G * (D + 2) * 4;
-  static constexpr int COMBINE_BYTES = kMaxSplits * G * 4 + 2 * G * 4;
-  static constexpr int SMEM = DATA_BYTES + 2 * NST * 8 + 16;
+  static constexpr int OFF_MERGE = DATA_BYTES;   // [NW][G][D] o, [NW][G] m, [NW][G] l
+  static constexpr int MERGE_BYTES = NW * G * (D + 2) * 4;
+  static constexpr int OFF_BAR = (OFF_MERGE + MERGE_BYTES + 15) / 16 * 16;
+  static constexpr int SMEM = OFF_BAR + 2 * NST * 8 + 32;
   static constexpr int THREADS = (NW + 1) * 32;
   static_assert(V % LPT == 0 && RP <= GP, "bad reduce-scatter shape");
-  static_assert(MERGE_BYTES <= DATA_BYTES && COMBINE_BYTES <= DATA_BYTES, "merge area");
+  static_assert(THREADS * 8 <= DATA_BYTES, "scan scratch");
 };
 
 // Copy rows [row0, row0 + cnt) of one region into shared memory; row xr (if
@@ -100,305 +101,388 @@ __device__ __forceinline__ void reduce_scatter(float (&x)[V], int c) {
   }
 }
 
+// Rows of item `id` (items are ordered b-major: the retrieval heads of a
+// sequence, then its streaming heads). Retrieval: t + 1 rows; streaming:
+// min(t + 1, S + W) ring rows; t = tokens held before this step.
+__device__ __forceinline__ int item_rows(const DecodeArgs& a, int id) {
+  const CacheGeom& g = a.geom;
+  const int HK = g.n_r + g.n_s;
+  const int b = id / HK, k = id - b * HK;
+  const int t = __ldcg(&a.lens[b]);
+  return k < g.n_r ? t + 1 : min(t + 1, g.S + g.W);
+}
+
+// CTA whose row range contains global row x (ranges [p*T/P, (p+1)*T/P)).
+__device__ __forceinline__ int cta_of(long long x, long long total, int P) {
+  return (int)(((x + 1) * (long long)P - 1) / total);
+}
+
 template <class C>
 __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constant__ DecodeArgs a) {
   constexpr int D = C::D, G = C::G, RB = C::RB, TOK = C::TOK, NST = C::NST;
   extern __shared__ __align__(1024) uint8_t smem[];
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::DATA_BYTES);
+  float* mo = reinterpret_cast<float*>(smem + C::OFF_MERGE);  // [NW][G][D]
+  float* mm = mo + C::NW * G * D;                              // [NW][G]
+  float* ml = mm + C::NW * G;                                  // [NW][G]
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* empty = full + NST;
-  int* flag = reinterpret_cast<int*>(empty + NST);
+  long long* sh64 = reinterpret_cast<long long*>(empty + NST);  // [0] total, [1] first offset
+  int* sh32 = reinterpret_cast<int*>(sh64 + 2);                 // [0] first item, [1] combine flag
+  volatile int* abort_flag = sh32 + 2;                          // set once any bounded wait gives up
 
   const CacheGeom& g = a.geom;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int HK = g.n_r + g.n_s;
+  const int n_items = g.B * HK;
+  const int P = a.n_ctas, p = blockIdx.x;
 
-  // ---- work unit
-  const int per_b = g.n_r * a.ns_r + g.n_s * a.ns_s;
-  const int b = blockIdx.x / per_b;
-  int rem = blockIdx.x - b * per_b;
-  int kind, hi, split, nsplit;
-  if (rem < g.n_r * a.ns_r) {
-    kind = 0; hi = rem / a.ns_r; split = rem - hi * a.ns_r; nsplit = a.ns_r;
-  } else {
-    rem -= g.n_r * a.ns_r;
-    kind = 1; hi = rem / a.ns_s; split = rem - hi * a.ns_s; nsplit = a.ns_s;
-  }
-  const int kvh = kind ? g.s_head[hi] : g.r_head[hi];
-  const int t = __ldcg(&a.lens[b]);  // position of the new token
-  int n, xr, cap;
-  if (kind == 0) {
-    cap = g.max_seq; n = t + 1; xr = t;
-  } else {
-    cap = g.S + g.W; n = min(t + 1, cap); xr = t < g.S ? t : g.S + (t - g.S) % g.W;
-  }
-  const int chunk = (n + nsplit - 1) / nsplit;
-  const int r_begin = min(n, split * chunk);
-  const int r_end = min(n, r_begin + chunk);
-  const int n_tiles = (r_end - r_begin + TOK - 1) / TOK;
-
-  const size_t reg = kind ? g.s_region(b, hi) : g.r_region(b, hi);
-  const uint8_t* Kc = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.kv) + reg);
-  const uint8_t* Vc = Kc + (size_t)cap * RB;
-  const size_t new_off = ((size_t)b * g.Hkv + kvh) * D;
-  const uint8_t* kn = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.k_new) + new_off);
-  const uint8_t* vn = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.v_new) + new_off);
-
-  if (threadIdx.x == 0) {
-#pragma unroll
-    for (int s = 0; s < NST; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], C::NW);
+  // ---- prefix sums of the items' rows: every CTA finds its share of the
+  // concatenated rows [p * total / P, (p + 1) * total / P) and the first item
+  // it touches. The ring memory is scratch here.
+  {
+    long long* part = reinterpret_cast<long long*>(smem);
+    const int per = (n_items + C::THREADS - 1) / C::THREADS;
+    const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
+    long long mine = 0;
+    for (int id = i0; id < i1; ++id) mine += item_rows(a, id);
+    part[threadIdx.x] = mine;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      long long run = 0;
+      for (int t = 0; t < C::THREADS; ++t) {
+        const long long v = part[t];
+        part[t] = run;
+        run += v;
+      }
+      sh64[0] = run;
+      sh32[0] = n_items;
+      sh64[1] = run;
     }
-    fence_mbar_init();
+    __syncthreads();
+    const long long total = sh64[0];
+    const long long start = (long long)p * total / P;
+    long long off = part[threadIdx.x];
+    if (i0 < i1 && off <= start && start < off + mine) {
+      int id = i0;
+      while (true) {
+        const int r = item_rows(a, id);
+        if (start < off + r) break;
+        off += r;
+        ++id;
+      }
+      sh32[0] = id;
+      sh64[1] = off;
+    }
+    if (threadIdx.x == 0) {
+#pragma unroll
+      for (int s = 0; s < NST; ++s) {
+        mbar_init(&full[s], 1);
+        mbar_init(&empty[s], C::NW);
+      }
+      *abort_flag = 0;
+      fence_mbar_init();
+    }
+    __syncthreads();
   }
-  __syncthreads();
-
-  float m[G], l[G];
-  float2 o[G][4];
-  const int gi = lane / C::LPT, c = lane % C::LPT;
-  const int grp = warp * C::GPW + gi;
+  const long long total = sh64[0];
+  const long long start = (long long)p * total / P;
+  const long long end = (long long)(p + 1) * total / P;
+  const int first_id = sh32[0];
+  const long long first_off = sh64[1];
 
   if (warp == C::NW) {
     // ------------------------------------------------------------ producer
-    if (xr >= r_begin && xr < r_end && lane < D / 8) {
-      uint8_t* Kw = const_cast<uint8_t*>(Kc);
-      uint8_t* Vw = const_cast<uint8_t*>(Vc);
-      reinterpret_cast<uint4*>(Kw + (size_t)xr * RB)[lane] = reinterpret_cast<const uint4*>(kn)[lane];
-      reinterpret_cast<uint4*>(Vw + (size_t)xr * RB)[lane] = reinterpret_cast<const uint4*>(vn)[lane];
-    }
-    if (lane == 0) {
-      int issued = 0;
-      for (int it = 0; it < n_tiles; ++it) {
-        const int st = it % NST;
-        const uint32_t ph = (it / NST) & 1;
-        if (it >= NST && !mbar_wait(&empty[st], ph ^ 1, a.err)) break;
-        const int row0 = r_begin + it * TOK;
-        const int cnt = min(TOK, r_end - row0);
-        mbar_arrive_expect_tx(&full[st], (uint32_t)cnt * RB * 2);
-        uint8_t* ks = smem + st * C::STAGE_BYTES;
-        copy_rows<RB>(ks, Kc, kn, row0, cnt, xr, &full[st]);
-        copy_rows<RB>(ks + TOK * RB, Vc, vn, row0, cnt, xr, &full[st]);
-        issued = it + 1;
+    int it = 0;
+    long long off = first_off;
+    for (int id = first_id; id < n_items && off < end; ++id) {
+      const int rows = item_rows(a, id);
+      const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
+      off += rows;
+      if (lo >= hi) continue;
+      const int b = id / HK, k = id - b * HK;
+      const int kind = k < g.n_r ? 0 : 1, hi_idx = kind ? k - g.n_r : k;
+      const int kvh = kind ? g.s_head[hi_idx] : g.r_head[hi_idx];
+      const int t = __ldcg(&a.lens[b]);
+      const int cap = kind ? g.S + g.W : g.max_seq;
+      const int xr = kind == 0 ? t : (t < g.S ? t : g.S + (t - g.S) % g.W);
+      const size_t reg = kind ? g.s_region(b, hi_idx) : g.r_region(b, hi_idx);
+      const uint8_t* Kc = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.kv) + reg);
+      const uint8_t* Vc = Kc + (size_t)cap * RB;
+      const size_t new_off = ((size_t)b * g.Hkv + kvh) * D;
+      const uint8_t* kn = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.k_new) + new_off);
+      const uint8_t* vn = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.v_new) + new_off);
+      if (xr >= lo && xr < hi && lane < D / 8) {
+        // append the new token (its row is read from the input below)
+        reinterpret_cast<uint4*>(const_cast<uint8_t*>(Kc) + (size_t)xr * RB)[lane] =
+            reinterpret_cast<const uint4*>(kn)[lane];
+        reinterpret_cast<uint4*>(const_cast<uint8_t*>(Vc) + (size_t)xr * RB)[lane] =
+            reinterpret_cast<const uint4*>(vn)[lane];
       }
-      // Every issued copy has landed before shared memory is reused (normally
-      // the consumers already waited for all of them).
-      for (int it = issued > NST ? issued - NST : 0; it < issued; ++it)
-        mbar_wait(&full[it % NST], (it / NST) & 1, a.err);
+      if (lane == 0) {
+        for (int row0 = lo; row0 < hi && !*abort_flag; row0 += TOK, ++it) {
+          const int st = it % NST;
+          if (it >= NST && !mbar_wait(&empty[st], ((it / NST) & 1) ^ 1, a.err)) {
+            *abort_flag = 1;
+            break;
+          }
+          const int cnt = min(TOK, hi - row0);
+          mbar_arrive_expect_tx(&full[st], (uint32_t)cnt * RB * 2);
+          uint8_t* ks = smem + st * C::STAGE_BYTES;
+          copy_rows<RB>(ks, Kc, kn, row0, cnt, xr, &full[st]);
+          copy_rows<RB>(ks + TOK * RB, Vc, vn, row0, cnt, xr, &full[st]);
+        }
+      }
+      __syncwarp();
     }
+    // every issued copy lands before the CTA can exit
+    if (lane == 0)
+      for (int j = it > NST ? it - NST : 0; j < it; ++j) mbar_wait(&full[j % NST], (j / NST) & 1, a.err);
   } else {
     // ------------------------------------------------------------ consumers
-    float2 qf[G][4];
-    const bf16* qb = static_cast<const bf16*>(a.q) + ((size_t)b * g.Hq + (size_t)kvh * G) * D + c * 8;
-#pragma unroll
-    for (int r = 0; r < G; ++r) {
-      const uint4 raw = *reinterpret_cast<const uint4*>(qb + (size_t)r * D);
-      qf[r][0] = bf16x2_to_float2(raw.x);
-      qf[r][1] = bf16x2_to_float2(raw.y);
-      qf[r][2] = bf16x2_to_float2(raw.z);
-      qf[r][3] = bf16x2_to_float2(raw.w);
-      m[r] = -INFINITY;
-      l[r] = 0.f;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) o[r][e] = make_float2(0.f, 0.f);
-    }
+    const int gi = lane / C::LPT, c = lane % C::LPT;
+    const int grp = warp * C::GPW + gi;
     const int tb = grp * C::NT;  // first tile row of this group
+    int it = 0;
+    long long off = first_off;
+    for (int id = first_id; id < n_items && off < end; ++id) {
+      const int rows = item_rows(a, id);
+      const long long item_off = off;
+      const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
+      off += rows;
+      if (lo >= hi) continue;
+      const int b = id / HK, k = id - b * HK;
+      const int kind = k < g.n_r ? 0 : 1;
+      const int kvh = kind ? g.s_head[k - g.n_r] : g.r_head[k];
 
-    for (int it = 0; it < n_tiles; ++it) {
-      const int st = it % NST;
-      const uint32_t ph = (it / NST) & 1;
-      if (!mbar_wait(&full[st], ph, a.err)) break;
-      const int cnt = min(TOK, r_end - (r_begin + it * TOK));
-      const uint8_t* ks = smem + st * C::STAGE_BYTES;
-      const uint8_t* vs = ks + TOK * RB;
-
-      // partial q.k over this lane's 8 d-elements, for NT rows x G heads
-      float part[C::V];
-      {
-        float2 kf[C::NT][4];
+      float2 qf[G][4];
+      float m[G], l[G];
+      float2 o[G][4];
+      const bf16* qb = static_cast<const bf16*>(a.q) + ((size_t)b * g.Hq + (size_t)kvh * G) * D + c * 8;
 #pragma unroll
-        for (int tt = 0; tt < C::NT; ++tt) {
-          const int row = min(tb + tt, cnt - 1);
-          const uint4 raw = lds128(ks + row * RB + c * 16);
-          kf[tt][0] = bf16x2_to_float2(raw.x);
-          kf[tt][1] = bf16x2_to_float2(raw.y);
-          kf[tt][2] = bf16x2_to_float2(raw.z);
-          kf[tt][3] = bf16x2_to_float2(raw.w);
+      for (int r = 0; r < G; ++r) {
+        const uint4 raw = *reinterpret_cast<const uint4*>(qb + (size_t)r * D);
+        qf[r][0] = bf16x2_to_float2(raw.x);
+        qf[r][1] = bf16x2_to_float2(raw.y);
+        qf[r][2] = bf16x2_to_float2(raw.z);
+        qf[r][3] = bf16x2_to_float2(raw.w);
+        m[r] = -INFINITY;
+        l[r] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[r][e] = make_float2(0.f, 0.f);
+      }
+
+      for (int row0 = lo; row0 < hi; row0 += TOK, ++it) {
+        const int st = it % NST;
+        // warp-uniform: every lane leaves the loop together if a wait gave up
+        bool stop = __any_sync(kFull, *abort_flag != 0);
+        if (!stop) stop = !__all_sync(kFull, mbar_wait(&full[st], (it / NST) & 1, a.err));
+        if (stop) {
+          *abort_flag = 1;
+          break;
         }
+        const int cnt = min(TOK, hi - row0);
+        const uint8_t* ks = smem + st * C::STAGE_BYTES;
+        const uint8_t* vs = ks + TOK * RB;
+
+        float part[C::V];
+        {
+          float2 kf[C::NT][4];
 #pragma unroll
-        for (int tt = 0; tt < C::NT; ++tt) {
+          for (int tt = 0; tt < C::NT; ++tt) {
+            const int row = min(tb + tt, cnt - 1);
+            const uint4 raw = lds128(ks + row * RB + c * 16);
+            kf[tt][0] = bf16x2_to_float2(raw.x);
+            kf[tt][1] = bf16x2_to_float2(raw.y);
+            kf[tt][2] = bf16x2_to_float2(raw.z);
+            kf[tt][3] = bf16x2_to_float2(raw.w);
+          }
 #pragma unroll
-          for (int r = 0; r < C::GP; ++r) {
-            if (r < G) {
-              float2 acc = make_float2(0.f, 0.f);
+          for (int tt = 0; tt < C::NT; ++tt) {
 #pragma unroll
-              for (int e = 0; e < 4; ++e) acc = __ffma2_rn(qf[r][e], kf[tt][e], acc);
-              part[tt * C::GP + r] = acc.x + acc.y;
-            } else {
-              part[tt * C::GP + r] = 0.f;
+            for (int r = 0; r < C::GP; ++r) {
+              if (r < G) {
+                float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc = __ffma2_rn(qf[r][e], kf[tt][e], acc);
+                part[tt * C::GP + r] = acc.x + acc.y;
+              } else {
+                part[tt * C::GP + r] = 0.f;
+              }
             }
           }
         }
-      }
-      reduce_scatter<C::LPT, C::V>(part, c);
+        reduce_scatter<C::LPT, C::V>(part, c);
 
-      // scores held by this lane: value v = c*RP + k -> row tt = v / GP, head r = v % GP
-      float s[C::RP], mx[C::RP];
+        float s[C::RP], mx[C::RP];
 #pragma unroll
-      for (int k = 0; k < C::RP; ++k) {
-        const int v = c * C::RP + k;
-        const int tt = v / C::GP, r = v % C::GP;
-        const bool valid = (tb + tt < cnt) && (r < G);
-        s[k] = valid ? part[k] * a.scale_log2 : -INFINITY;
-        mx[k] = s[k];
-      }
+        for (int kk = 0; kk < C::RP; ++kk) {
+          const int v = c * C::RP + kk;
+          const int tt = v / C::GP, r = v % C::GP;
+          const bool valid = (tb + tt < cnt) && (r < G);
+          s[kk] = valid ? part[kk] * a.scale_log2 : -INFINITY;
+          mx[kk] = s[kk];
+        }
 #pragma unroll
-      for (int msk = C::Q; msk < C::LPT; msk *= 2)
+        for (int msk = C::Q; msk < C::LPT; msk *= 2)
 #pragma unroll
-        for (int k = 0; k < C::RP; ++k) mx[k] = fmaxf(mx[k], __shfl_xor_sync(kFull, mx[k], msk));
-      float bm[G];
+          for (int kk = 0; kk < C::RP; ++kk) mx[kk] = fmaxf(mx[kk], __shfl_xor_sync(kFull, mx[kk], msk));
+        float bm[G];
 #pragma unroll
-      for (int j = 0; j < C::Q; ++j)
+        for (int j = 0; j < C::Q; ++j)
 #pragma unroll
-        for (int k = 0; k < C::RP; ++k)
-          if (j * C::RP + k < G) bm[j * C::RP + k] = __shfl_sync(kFull, mx[k], gi * C::LPT + j);
+          for (int kk = 0; kk < C::RP; ++kk)
+            if (j * C::RP + kk < G) bm[j * C::RP + kk] = __shfl_sync(kFull, mx[kk], gi * C::LPT + j);
 
-      bool need = false;
+        bool need = false;
 #pragma unroll
-      for (int r = 0; r < G; ++r) need |= bm[r] > m[r] + kRescaleThreshold;
-      if (__any_sync(kFull, need)) {
+        for (int r = 0; r < G; ++r) need |= bm[r] > m[r] + kRescaleThreshold;
+        if (__any_sync(kFull, need)) {
 #pragma unroll
-        for (int r = 0; r < G; ++r) {
-          const float mn = fmaxf(m[r], bm[r]);
-          const float alpha = (m[r] == -INFINITY) ? 0.f : fast_exp2(m[r] - mn);
-          m[r] = mn;
-          l[r] *= alpha;
+          for (int r = 0; r < G; ++r) {
+            const float mn = fmaxf(m[r], bm[r]);
+            const float alpha = (m[r] == -INFINITY) ? 0.f : fast_exp2(m[r] - mn);
+            m[r] = mn;
+            l[r] *= alpha;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            o[r][e].x *= alpha;
-            o[r][e].y *= alpha;
+            for (int e = 0; e < 4; ++e) {
+              o[r][e].x *= alpha;
+              o[r][e].y *= alpha;
+            }
+          }
+        }
+
+        float pr[C::RP];
+#pragma unroll
+        for (int kk = 0; kk < C::RP; ++kk) {
+          const int r = (c % C::Q) * C::RP + kk;
+          float mr = m[0];
+#pragma unroll
+          for (int rr = 1; rr < G; ++rr) mr = (rr == r) ? m[rr] : mr;
+          pr[kk] = (s[kk] == -INFINITY) ? 0.f : fast_exp2(s[kk] - mr);
+        }
+
+        float2 vf[C::NT][4];
+#pragma unroll
+        for (int tt = 0; tt < C::NT; ++tt) {
+          const int row = min(tb + tt, cnt - 1);
+          const uint4 raw = lds128(vs + row * RB + c * 16);
+          vf[tt][0] = bf16x2_to_float2(raw.x);
+          vf[tt][1] = bf16x2_to_float2(raw.y);
+          vf[tt][2] = bf16x2_to_float2(raw.z);
+          vf[tt][3] = bf16x2_to_float2(raw.w);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+
+#pragma unroll
+        for (int tt = 0; tt < C::NT; ++tt) {
+#pragma unroll
+          for (int r = 0; r < G; ++r) {
+            const int v = tt * C::GP + r;
+            const float pv = __shfl_sync(kFull, pr[v % C::RP], gi * C::LPT + v / C::RP);
+            l[r] += pv;
+            const float2 pp = make_float2(pv, pv);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) o[r][e] = __ffma2_rn(pp, vf[tt][e], o[r][e]);
           }
         }
       }
 
-      float p[C::RP];
+      // ---- merge the groups of each warp with shuffles, then the warps
 #pragma unroll
-      for (int k = 0; k < C::RP; ++k) {
-        const int r = (c % C::Q) * C::RP + k;
-        float mr = m[0];
-#pragma unroll
-        for (int rr = 1; rr < G; ++rr) mr = (rr == r) ? m[rr] : mr;
-        p[k] = (s[k] == -INFINITY) ? 0.f : fast_exp2(s[k] - mr);
-      }
-
-      float2 vf[C::NT][4];
-#pragma unroll
-      for (int tt = 0; tt < C::NT; ++tt) {
-        const int row = min(tb + tt, cnt - 1);
-        const uint4 raw = lds128(vs + row * RB + c * 16);
-        vf[tt][0] = bf16x2_to_float2(raw.x);
-        vf[tt][1] = bf16x2_to_float2(raw.y);
-        vf[tt][2] = bf16x2_to_float2(raw.z);
-        vf[tt][3] = bf16x2_to_float2(raw.w);
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[st]);
-
-#pragma unroll
-      for (int tt = 0; tt < C::NT; ++tt) {
+      for (int msk = C::LPT; msk < 32; msk *= 2) {
 #pragma unroll
         for (int r = 0; r < G; ++r) {
-          const int v = tt * C::GP + r;
-          const float pv = __shfl_sync(kFull, p[v % C::RP], gi * C::LPT + v / C::RP);
-          l[r] += pv;
-          const float2 pp = make_float2(pv, pv);
+          const float m_o = __shfl_xor_sync(kFull, m[r], msk);
+          const float l_o = __shfl_xor_sync(kFull, l[r], msk);
+          const float M = fmaxf(m[r], m_o);
+          const float wa = (m[r] == -INFINITY) ? 0.f : fast_exp2(m[r] - M);
+          const float wb = (m_o == -INFINITY) ? 0.f : fast_exp2(m_o - M);
+          l[r] = l[r] * wa + l_o * wb;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) o[r][e] = __ffma2_rn(pp, vf[tt][e], o[r][e]);
+          for (int e = 0; e < 4; ++e) {
+            const float ox = __shfl_xor_sync(kFull, o[r][e].x, msk);
+            const float oy = __shfl_xor_sync(kFull, o[r][e].y, msk);
+            o[r][e].x = o[r][e].x * wa + ox * wb;
+            o[r][e].y = o[r][e].y * wa + oy * wb;
+          }
+          m[r] = M;
         }
       }
-    }
-  }
-
-  // ---- merge the groups of this CTA (stage memory is free now)
-  __syncthreads();
-  float* mo = reinterpret_cast<float*>(smem);           // [NG][G][D]
-  float* mm = mo + C::NG * G * D;                        // [NG][G]
-  float* ml = mm + C::NG * G;                            // [NG][G]
-  if (warp < C::NW) {
+      if (gi == 0) {
 #pragma unroll
-    for (int r = 0; r < G; ++r) {
-      float* dst = mo + ((size_t)grp * G + r) * D + c * 8;
+        for (int r = 0; r < G; ++r) {
+          float* dst = mo + ((size_t)warp * G + r) * D + c * 8;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) *reinterpret_cast<float2*>(dst + 2 * e) = o[r][e];
-      if (c == 0) {
-        mm[grp * G + r] = m[r];
-        ml[grp * G + r] = l[r];
+          for (int e = 0; e < 4; ++e) *reinterpret_cast<float2*>(dst + 2 * e) = o[r][e];
+          if (c == 0) {
+            mm[warp * G + r] = m[r];
+            ml[warp * G + r] = l[r];
+          }
+        }
       }
-    }
-  }
-  __syncthreads();
+      named_barrier_sync(1, C::NW * 32);
 
-  const bool single = nsplit == 1;
-  float* part_base = a.partials + (((size_t)b * g.Hkv + kvh) * a.split_stride + split) * (size_t)(G * (D + 2));
-  bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * D;
-  for (int idx = threadIdx.x; idx < G * D; idx += C::THREADS) {
-    const int r = idx / D, d = idx - r * D;
-    float M = -INFINITY;
-#pragma unroll
-    for (int q = 0; q < C::NG; ++q) M = fmaxf(M, mm[q * G + r]);
-    float O = 0.f, L = 0.f;
-#pragma unroll
-    for (int q = 0; q < C::NG; ++q) {
-      const float mq = mm[q * G + r];
-      const float w = (mq == -INFINITY) ? 0.f : fast_exp2(mq - M);
-      O += w * mo[((size_t)q * G + r) * D + d];
-      L += w * ml[q * G + r];
-    }
-    if (single) {
-      outp[idx] = __float2bfloat16_rn(O / L);
-    } else {
-      __stcg(part_base + idx, O);
-      if (d == 0) {
-        __stcg(part_base + G * D + r, M);
-        __stcg(part_base + G * D + G + r, L);
-      }
-    }
-  }
-
-  if (!single) {
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      const uint32_t prev = atomicAdd(&a.counters[b * g.Hkv + kvh], 1u);
-      *flag = (prev == (uint32_t)nsplit - 1u);
-    }
-    __syncthreads();
-    if (*flag) {
-      __threadfence();
-      // last split to finish: merge all partials of (b, head)
-      float* wts = reinterpret_cast<float*>(smem);  // [nsplit][G]
-      float* Ls = wts + kMaxSplits * G;             // [G]
-      const float* pb0 = a.partials + ((size_t)b * g.Hkv + kvh) * a.split_stride * (size_t)(G * (D + 2));
-      if (threadIdx.x < G) {
-        const int r = threadIdx.x;
+      const int f = cta_of(item_off, total, P), lst = cta_of(item_off + rows - 1, total, P);
+      const bool single = f == lst;
+      const int slot = (p == f) ? 1 : 0;
+      float* pbase = a.partials + ((size_t)p * 2 + slot) * (size_t)(G * (D + 2));
+      bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * D;
+      for (int idx = threadIdx.x; idx < G * D; idx += C::NW * 32) {
+        const int r = idx / D, d = idx - r * D;
         float M = -INFINITY;
-        for (int sp = 0; sp < nsplit; ++sp) M = fmaxf(M, __ldcg(pb0 + (size_t)sp * G * (D + 2) + G * D + r));
-        float L = 0.f;
-        for (int sp = 0; sp < nsplit; ++sp) {
-          const float* pb = pb0 + (size_t)sp * G * (D + 2);
-          const float ms = __ldcg(pb + G * D + r);
-          const float w = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
-          wts[sp * G + r] = w;
-          L += w * __ldcg(pb + G * D + G + r);
+#pragma unroll
+        for (int w = 0; w < C::NW; ++w) M = fmaxf(M, mm[w * G + r]);
+        float O = 0.f, L = 0.f;
+#pragma unroll
+        for (int w = 0; w < C::NW; ++w) {
+          const float mw = mm[w * G + r];
+          const float wt = (mw == -INFINITY) ? 0.f : fast_exp2(mw - M);
+          O += wt * mo[((size_t)w * G + r) * D + d];
+          L += wt * ml[w * G + r];
         }
-        Ls[r] = L;
+        if (single) {
+          outp[idx] = __float2bfloat16_rn(O / L);
+        } else {
+          __stcg(pbase + idx, O);
+          if (d == 0) {
+            __stcg(pbase + G * D + r, M);
+            __stcg(pbase + G * D + G + r, L);
+          }
+        }
       }
-      __syncthreads();
-      for (int idx = threadIdx.x; idx < G * D; idx += C::THREADS) {
-        const int r = idx / D;
-        float O = 0.f;
-        for (int sp = 0; sp < nsplit; ++sp) O += wts[sp * G + r] * __ldcg(pb0 + (size_t)sp * G * (D + 2) + idx);
-        outp[idx] = __float2bfloat16_rn(O / Ls[r]);
+      if (!single) {
+        __threadfence();
+        named_barrier_sync(1, C::NW * 32);
+        if (threadIdx.x == 0) {
+          const uint32_t prev = atomicAdd(&a.counters[id], 1u);
+          sh32[1] = (prev == (uint32_t)(lst - f));
+        }
+        named_barrier_sync(1, C::NW * 32);
+        if (sh32[1]) {
+          // last part of this item to finish: merge the parts of CTAs f..lst
+          __threadfence();
+          for (int idx = threadIdx.x; idx < G * D; idx += C::NW * 32) {
+            const int r = idx / D;
+            float M = -INFINITY;
+            for (int q = f; q <= lst; ++q) {
+              const float* pb = a.partials + ((size_t)q * 2 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
+              M = fmaxf(M, __ldcg(pb + G * D + r));
+            }
+            float O = 0.f, L = 0.f;
+            for (int q = f; q <= lst; ++q) {
+              const float* pb = a.partials + ((size_t)q * 2 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
+              const float mq = __ldcg(pb + G * D + r);
+              const float wt = (mq == -INFINITY) ? 0.f : fast_exp2(mq - M);
+              O += wt * __ldcg(pb + idx);
+              L += wt * __ldcg(pb + G * D + G + r);
+            }
+            outp[idx] = __float2bfloat16_rn(O / L);
+          }
+          if (threadIdx.x == 0) a.counters[id] = 0u;
+        }
       }
-      if (threadIdx.x == 0) a.counters[b * g.Hkv + kvh] = 0u;
+      named_barrier_sync(1, C::NW * 32);
     }
   }
 
@@ -416,7 +500,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
 }
 
 template <int D, int G>
-cudaError_t launch_cfg(const DecodeArgs& a, int n_ctas, cudaStream_t s) {
+cudaError_t launch_cfg(const DecodeArgs& a, cudaStream_t s) {
   using C = DecodeCfg<D, G>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -424,7 +508,7 @@ cudaError_t launch_cfg(const DecodeArgs& a, int n_ctas, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  decode_kernel<C><<<n_ctas, C::THREADS, C::SMEM, s>>>(a);
+  decode_kernel<C><<<a.n_ctas, C::THREADS, C::SMEM, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -435,23 +519,34 @@ bool decode_supported(int D, int G) {
   return G == 1 || G == 2 || G == 4 || G == 7 || G == 8;
 }
 
-cudaError_t launch_decode(const DecodeArgs& a, int n_ctas, cudaStream_t s) {
+// Two CTAs fit on an SM (about 100 KB of shared memory each), so 2 x SMs
+// CTAs run as one wave; small launches use fewer, at least 256 rows each.
+int decode_ctas(long long total_rows, int num_sms) {
+  const long long by_rows = (total_rows + 255) / 256;
+  long long p = 2LL * num_sms;
+  if (by_rows < p) p = by_rows;
+  return p < 1 ? 1 : (int)p;
+}
+
+size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 2 * G * (D + 2); }
+
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;
   if (D == 128) {
     switch (G) {
-      case 1: return launch_cfg<128, 1>(a, n_ctas, s);
-      case 2: return launch_cfg<128, 2>(a, n_ctas, s);
-      case 4: return launch_cfg<128, 4>(a, n_ctas, s);
-      case 7: return launch_cfg<128, 7>(a, n_ctas, s);
-      case 8: return launch_cfg<128, 8>(a, n_ctas, s);
+      case 1: return launch_cfg<128, 1>(a, s);
+      case 2: return launch_cfg<128, 2>(a, s);
+      case 4: return launch_cfg<128, 4>(a, s);
+      case 7: return launch_cfg<128, 7>(a, s);
+      case 8: return launch_cfg<128, 8>(a, s);
     }
   } else if (D == 64) {
     switch (G) {
-      case 1: return launch_cfg<64, 1>(a, n_ctas, s);
-      case 2: return launch_cfg<64, 2>(a, n_ctas, s);
-      case 4: return launch_cfg<64, 4>(a, n_ctas, s);
-      case 7: return launch_cfg<64, 7>(a, n_ctas, s);
-      case 8: return launch_cfg<64, 8>(a, n_ctas, s);
+      case 1: return launch_cfg<64, 1>(a, s);
+      case 2: return launch_cfg<64, 2>(a, s);
+      case 4: return launch_cfg<64, 4>(a, s);
+      case 7: return launch_cfg<64, 7>(a, s);
+      case 8: return launch_cfg<64, 8>(a, s);
     }
   }
   return cudaErrorInvalidValue;

@@ -125,21 +125,14 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   e = cudaMemsetAsync(header, 0, (size_t)(64 + items) * 4, s);
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaMemsetAsync failed");
 
-  // Split schedule as the handle API computes it, bounded by the partial space.
-  const size_t per_split = (size_t)items * G * (c.d_head + 2) * 4;
-  int stride = (int)(kNoAllocPartialBytes / per_split);
-  if (stride > kMaxSplits) stride = kMaxSplits;
-  if (stride < 1) stride = 1;
-  const int maxlen = max_len + 1;
-  const int win = maxlen < c.sink + c.window ? maxlen : c.sink + c.window;
-  const double total = (double)c.batch * ((double)n_r * maxlen + (double)n_s * win);
-  const double target = (double)num_sms * 2 * 4;
-  int chunk = (int)(total / target + 0.999999);
-  if (chunk < 512) chunk = 512;
-  int ns_r = n_r ? (maxlen + chunk - 1) / chunk : 0;
-  int ns_s = n_s ? (win + chunk - 1) / chunk : 0;
-  if (n_r) ns_r = ns_r < 1 ? 1 : (ns_r > stride ? stride : ns_r);
-  if (n_s) ns_s = ns_s < 1 ? 1 : (ns_s > stride ? stride : ns_s);
+  // CTA count as the handle API computes it (from an upper bound of the rows),
+  // bounded by the partial space.
+  const long long t1 = (long long)max_len + 1;
+  const long long win = t1 < c.sink + c.window ? t1 : c.sink + c.window;
+  const long long total = (long long)c.batch * ((long long)n_r * t1 + (long long)n_s * win);
+  int n_ctas = decode_ctas(total, num_sms);
+  const int cap_ctas = (int)(kNoAllocPartialBytes / (decode_partial_floats(1, G, c.d_head) * 4));
+  if (n_ctas > cap_ctas) n_ctas = cap_ctas;
 
   DecodeArgs a;
   a.geom = g;
@@ -153,11 +146,9 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   a.done = header + 32;
   a.counters = header + 64;
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
-  a.ns_r = ns_r;
-  a.ns_s = ns_s;
-  a.split_stride = stride;
+  a.n_ctas = n_ctas;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));
-  e = launch_decode(a, c.batch * (n_r * ns_r + n_s * ns_s), s);
+  e = launch_decode(a, s);
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: kernel launch failed");
   return AOH_OK;
 }

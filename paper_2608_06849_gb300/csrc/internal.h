@@ -9,7 +9,6 @@
 namespace aoh {
 
 constexpr int kMaxKvHeads = 64;
-constexpr int kMaxSplits = 64;  // split-KV partials per (sequence, KV head)
 
 // Cache geometry as the kernels see it. Offsets are in bf16 elements from the
 // cache base; see include/aoh.h for the layout.
@@ -44,12 +43,11 @@ struct DecodeArgs {
   void* out;          // [B][Hq][D]
   void* kv;           // cache base
   int32_t* lens;      // [B] tokens held before this step (device)
-  float* partials;    // [B][Hkv][split_stride][G][D + 2]
-  uint32_t* counters; // [B][Hkv] split arrivals
+  float* partials;    // [n_ctas][2][G][D + 2]: a CTA's first and last shared item
+  uint32_t* counters; // [B][n_r + n_s] arrivals per item (items b-major, retrieval first)
   uint32_t* done;     // CTAs finished in this launch
   uint32_t* err;      // error word
-  int ns_r, ns_s;     // splits per retrieval / streaming head
-  int split_stride;   // partial slots per (b, head) in `partials`, >= ns_r, ns_s
+  int n_ctas;         // CTAs sharing the rows of all items equally
   float scale_log2;   // log2(e) / sqrt(D)
 };
 
@@ -82,7 +80,11 @@ void record_error(const char* msg);
 // Launchers (return the launch's cudaError_t).
 bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const void* v, int B, int T);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
-cudaError_t launch_decode(const DecodeArgs& a, int n_ctas, cudaStream_t s);
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
+// CTAs for a decode launch over `total_rows` cached rows on `num_sms` SMs.
+int decode_ctas(long long total_rows, int num_sms);
+// Floats of the partial buffer for `n_ctas` CTAs.
+size_t decode_partial_floats(int n_ctas, int G, int D);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
 bool decode_supported(int D, int G);
 

@@ -43,12 +43,12 @@ struct PfCfg {
   static constexpr int BOX = 128 * 64 * 2;       // bytes of one [128 rows][64] box
   static constexpr int QBYTES = DBLK * BOX;
   static constexpr int KVBYTES = DBLK * BOX;
-  static constexpr int PBYTES = 2 * BOX;         // [128 rows][128 keys]
+  static constexpr int PBYTES = 2 * BOX;         // one P buffer: [128 rows][128 keys]
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_KV = OFF_Q + QBYTES;
   static constexpr int OFF_P = OFF_KV + kNS * KVBYTES;
-  static constexpr int OFF_BAR = OFF_P + PBYTES;
-  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 1 + 1 + 1;
+  static constexpr int OFF_BAR = OFF_P + 2 * PBYTES;
+  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 1 + 2 + 1;
   static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;
   static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, false);
   static constexpr uint32_t IDESC_PV = idesc_bf16(kBM, D, true);
@@ -83,8 +83,8 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
   uint64_t* s_full = kv_empty + kNS;
   uint64_t* s_empty = s_full + 2;
   uint64_t* p_full = s_empty + 2;
-  uint64_t* pv_done = p_full + 1;
-  uint64_t* drain = pv_done + 1;
+  uint64_t* pv_done = p_full + 1;  // [2]: PV of tile x completes pv_done[x & 1]
+  uint64_t* drain = pv_done + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -119,7 +119,8 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       mbar_init(&s_empty[s], 4);
     }
     mbar_init(p_full, 4);
-    mbar_init(pv_done, 1);
+    mbar_init(&pv_done[0], 1);
+    mbar_init(&pv_done[1], 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -175,13 +176,14 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
         if (!wait_bar(p_full, x & 1, a.err, abort_flag)) return false;
         tc_fence_after();
         const uint32_t v_addr = kv_addr + st * C::KVBYTES;
+        const uint32_t pb = p_addr + (x & 1) * C::PBYTES;
 #pragma unroll
         for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(p_addr + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
+          const uint64_t ad = sdesc_sw128(pb + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
           const uint64_t bd = sdesc_sw128(v_addr + kk * 16 * 128, C::BOX, 1024);
           tc_mma(tmem + 256, ad, bd, C::IDESC_PV, (x > 0 || kk > 0) ? 1u : 0u);
         }
-        tc_commit(pv_done);
+        tc_commit(&pv_done[x & 1]);
         tc_commit(&kv_empty[st]);
         return true;
       };
@@ -225,36 +227,47 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       }
       tc_fence_after();
       float s[kBN];
-#pragma unroll
-      for (int c = 0; c < kBN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tl + (jj & 1) * 128 + c * 32, v);
+      {
+        uint32_t v0[32], v1[32], v2[32], v3[32];
+        const uint32_t sb = tl + (jj & 1) * 128;
+        tmem_ld32(sb, v0);
+        tmem_ld32(sb + 32, v1);
+        tmem_ld32(sb + 64, v2);
+        tmem_ld32(sb + 96, v3);
         tmem_ld_wait();
 #pragma unroll
-        for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(v[e]);
+        for (int e = 0; e < 32; ++e) {
+          s[e] = __uint_as_float(v0[e]);
+          s[32 + e] = __uint_as_float(v1[e]);
+          s[64 + e] = __uint_as_float(v2[e]);
+          s[96 + e] = __uint_as_float(v3[e]);
+        }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_empty[jj & 1]);
 
+      // hidden keys -> -inf. In tile coordinates key k is visible iff
+      // k <= kmax (causal and inside the sequence) and, for a streaming head,
+      // k < ks (a sink) or k >= kw (inside the window).
       const int jl = j0 + kBN - 1;
       const bool full_vis = jl <= q0 && jl < len && (!streaming || jl < S || (q0 + kBM - 1) - j0 < W);
-      float rmax = -INFINITY;
-      if (full_vis) {
+      if (!full_vis) {
+        const int kmax = min(i, len - 1) - j0;
+        const int ks = streaming ? S - j0 : kBN;
+        const int kw = streaming ? i - W + 1 - j0 : 0;
 #pragma unroll
-        for (int k = 0; k < kBN; ++k) {
-          s[k] *= a.scale_log2;
-          rmax = fmaxf(rmax, s[k]);
-        }
-      } else {
-#pragma unroll
-        for (int k = 0; k < kBN; ++k) {
-          const int jp = j0 + k;
-          const bool vis = jp <= i && jp < len && (!streaming || jp < S || i - jp < W);
-          s[k] = vis ? s[k] * a.scale_log2 : -INFINITY;
-          rmax = fmaxf(rmax, s[k]);
-        }
+        for (int k = 0; k < kBN; ++k) s[k] = (k <= kmax && (k < ks || k >= kw)) ? s[k] : -INFINITY;
       }
+      // row max of the raw scores (the scale is positive) in 8 chains
+      float mx8[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mx8[u] = s[u];
+#pragma unroll
+      for (int k = 8; k < kBN; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], s[k]);
+      const float rmax = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) *
+                         a.scale_log2;
       const float mn = fmaxf(m, rmax);
       const bool resc = mn > m + kRescaleThreshold;
       float alpha = 1.f;
@@ -263,52 +276,62 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
         m = mn;
       }
       const bool warp_resc = __any_sync(0xffffffffu, resc) && jj > 0;
-      float sum = 0.f;
-      uint32_t pk[kBN / 2];
-#pragma unroll
-      for (int k = 0; k < kBN; k += 2) {
-        const float p0 = (s[k] == -INFINITY) ? 0.f : fast_exp2(s[k] - m);
-        const float p1 = (s[k + 1] == -INFINITY) ? 0.f : fast_exp2(s[k + 1] - m);
-        sum += p0 + p1;
-        pk[k / 2] = float2_to_bf16x2(p0, p1);
+      const float neg_m = (m == -INFINITY) ? 0.f : -m;
+
+      // the P buffer of this tile was last read by PV of tile jj - 2
+      if (jj >= 2 && !__all_sync(0xffffffffu, wait_bar(&pv_done[jj & 1], ((jj - 2) >> 1) & 1, a.err, abort_flag))) {
+        ok = false;
+        break;
       }
+      // p = 2^(s * scale - m): one FFMA + one EX2 per element, hidden keys give
+      // 0; row sum in 8 chains; bf16 P straight into the swizzled K-major tile
+      uint8_t* prow = sP + (jj & 1) * C::PBYTES + r * 128;
+      float sum8[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) sum8[u] = 0.f;
+#pragma unroll
+      for (int ch = 0; ch < kBN / 8; ++ch) {
+        uint32_t w[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int k = ch * 8 + 2 * t;
+          const float p0 = fast_exp2(fmaf(s[k], a.scale_log2, neg_m));
+          const float p1 = fast_exp2(fmaf(s[k + 1], a.scale_log2, neg_m));
+          sum8[(ch * 4 + t) & 7] += p0 + p1;
+          w[t] = float2_to_bf16x2(p0, p1);
+        }
+        // key block ch / 8 (64 keys), 16-byte chunk ch % 8 of the 128-byte row
+        *reinterpret_cast<uint4*>(prow + (ch >> 3) * C::BOX + (((ch & 7) ^ (r & 7)) << 4)) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
       l = l * alpha + sum;
 
-      if (jj >= 1) {
-        if (!__all_sync(0xffffffffu, wait_bar(pv_done, (jj - 1) & 1, a.err, abort_flag))) {
+      // rescale O (rare): PV of tile jj - 1 must have landed first
+      if (warp_resc) {
+        if (!__all_sync(0xffffffffu, wait_bar(&pv_done[(jj - 1) & 1], ((jj - 1) >> 1) & 1, a.err, abort_flag))) {
           ok = false;
           break;
         }
         tc_fence_after();
-        if (warp_resc) {
 #pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t v[32];
-            tmem_ld32(tl + 256 + c * 32, v);
-            tmem_ld_wait();
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tl + 256 + c * 32, v);
+          tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-            tmem_st32(tl + 256 + c * 32, v);
-          }
-          tmem_st_wait();
+          for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+          tmem_st32(tl + 256 + c * 32, v);
         }
-      }
-      // P row r -> swizzled K-major tile: key block kb (64 keys), chunk c (8 keys)
-#pragma unroll
-      for (int kb = 0; kb < 2; ++kb) {
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int base = kb * 32 + c * 4;
-          uint4 val = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
-          *reinterpret_cast<uint4*>(sP + kb * C::BOX + r * 128 + ((c ^ (r & 7)) << 4)) = val;
-        }
+        tmem_st_wait();
       }
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);
     }
-    if (ok && __all_sync(0xffffffffu, wait_bar(pv_done, (n_tiles - 1) & 1, a.err, abort_flag))) {
+    if (ok && __all_sync(0xffffffffu,
+                         wait_bar(&pv_done[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1, a.err, abort_flag))) {
       tc_fence_after();
       const float inv = 1.f / l;
       bf16* op = static_cast<bf16*>(a.out) + (((size_t)b * a.T + min(i, len - 1)) * g.Hq + h) * D;
