@@ -144,37 +144,71 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
+# ------------------------------------------------------------------- ranks
+
+class Ranks:
+    """One process per GPU (torchrun env). The ranks run independent replicas
+    of the per-GPU workload; nothing crosses ranks on the data path. The only
+    collectives are the timing barrier and the max / sum over ranks."""
+
+    def __init__(self, backend="nccl"):
+        import torch.distributed as dist
+        self.dist = dist
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.backend = backend
+        if self.world > 1 and not dist.is_initialized():
+            dist.init_process_group(backend)
+
+    def _device(self):
+        return "cuda" if self.backend == "nccl" else "cpu"
+
+    def barrier(self):
+        import torch
+        if self.world > 1:
+            self.dist.barrier()
+        if self.backend == "nccl":
+            torch.cuda.synchronize()
+
+    def _reduce(self, x, op):
+        if self.world == 1:
+            return float(x)
+        import torch
+        t = torch.tensor([float(x)], dtype=torch.float64, device=self._device())
+        self.dist.all_reduce(t, op=op)
+        return float(t.item())
+
+    def max(self, x):
+        return self._reduce(x, self.dist.ReduceOp.MAX)
+
+    def sum(self, x):
+        return self._reduce(x, self.dist.ReduceOp.SUM)
+
+
+def replica_seed(base, rank):
+    """Each rank's replica draws its own inputs."""
+    return int(base) + 1000 * int(rank)
+
+
 # -------------------------------------------------------------- native arm
 
 def run_native(args):
     import torch
-    import torch.distributed as dist
 
     from paper_2608_06849_gb300 import aoh
     from paper_2608_06849_gb300 import build as aoh_build
     from paper_2608_06849_gb300.workloads import decode_inputs, randn_bf16
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1:
-        dist.init_process_group("nccl")
     torch.cuda.set_device(local)
+    ranks = Ranks("nccl")
+    world, rank = ranks.world, ranks.rank
     aoh_build.build()
     aoh.load()
     peaks, peak_note = load_peaks()
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    barrier = ranks.barrier
+    max_over_ranks = ranks.max
 
     stream = torch.cuda.current_stream()
     K, W = args.steps, args.warmup
@@ -184,8 +218,8 @@ def run_native(args):
     B, D, T0 = wl.batch, wl.d_head, wl.prefill_len
     total_steps = W + K + K + 2   # warmup, timed, e2e
     cache = aoh.Cache(B, wl.n_q_heads, wl.n_kv_heads, D, T0 + total_steps + 8, wl.sink, wl.window, labels)
-    kfill = randn_bf16((B, T0, wl.n_kv_heads, D), 7001 + rank, "cuda")
-    vfill = randn_bf16((B, T0, wl.n_kv_heads, D), 7002 + rank, "cuda")
+    kfill = randn_bf16((B, T0, wl.n_kv_heads, D), replica_seed(7001, rank), "cuda")
+    vfill = randn_bf16((B, T0, wl.n_kv_heads, D), replica_seed(7002, rank), "cuda")
     cache.prefill(None, kfill, vfill, None)
     torch.cuda.synchronize()
     del kfill, vfill
@@ -212,7 +246,8 @@ def run_native(args):
     cache.check()
     dec_us_step = dec_ms * 1000.0 / K
     avg_bytes = sum(step_bytes) / K
-    dec_gbs = avg_bytes / (dec_us_step * 1e-6) / 1e9
+    dec_gbs = avg_bytes / (dec_us_step * 1e-6) / 1e9          # per GPU (the roofline is per GPU)
+    dec_gbs_total = ranks.sum(avg_bytes) / (dec_us_step * 1e-6) / 1e9
 
     # e2e: same decode step through the C ABI from pinned host buffers
     hq = [t.cpu().pin_memory() for t in inputs[W]]
@@ -261,6 +296,7 @@ def run_native(args):
     pcache.check()
     flops = prefill_flops(pwl, plabels, T)
     pre_tflops = flops / (pre_ms * 1e-3) / 1e12
+    pre_tflops_total = ranks.sum(flops) / (pre_ms * 1e-3) / 1e12
     pcache.close()
 
     # ---------------- cpu baseline (oracle on a bounded sample), rank 0 only
@@ -294,11 +330,13 @@ def run_native(args):
             "parallelism": f"replicas x{world}",
         },
         "decode": {"us_per_step": round(dec_us_step, 3), "hbm_gbs": round(dec_gbs, 1),
+                   "hbm_gbs_all_ranks": round(dec_gbs_total, 1),
                    "bytes_per_step": int(avg_bytes), "kernel_us_median": round(statistics.median(per_step_ms) * 1000, 3)},
         "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                      "frac": round(dec_gbs / hbm_peak, 4), "traffic": traffic_for("decode"),
                      "peak_note": f"{peak_note} HBM copy bandwidth; kernel: decode split-KV"},
         "prefill": {"ms": round(pre_ms, 3), "tflops": round(pre_tflops, 2), "flops": flops, "steps": Kp,
+                    "tflops_all_ranks": round(pre_tflops_total, 2),
                     "roofline": {"bound": "tensor", "achieved": round(pre_tflops, 2), "peak": tf_peak,
                                  "unit": "TFLOP/s", "frac": round(pre_tflops / tf_peak, 4),
                                  "traffic": traffic_for("prefill"),
