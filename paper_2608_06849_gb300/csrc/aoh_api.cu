@@ -61,11 +61,11 @@ aoh_status check_config(const aoh_config* cfg, const uint8_t* labels, int* n_r, 
   return AOH_OK;
 }
 
-// Prefill tiles: one item per (b, query head, 128-row query tile), with the
+// Prefill work: one item per (b, query head, 128-row query tile), with the
 // number of 128-key tiles it visits as its cost; heaviest first so the
 // hardware block scheduler fills the machine longest-processing-time first.
 std::vector<int4> prefill_schedule(const CacheGeom& g, const std::vector<int32_t>& lens) {
-  constexpr int BM = 128, BN = 128;
+  constexpr int BM = 256, BN = 128;
   std::vector<int4> items;
   for (int b = 0; b < g.B; ++b) {
     for (int h = 0; h < g.Hq; ++h) {

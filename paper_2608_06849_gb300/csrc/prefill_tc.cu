@@ -1,26 +1,37 @@
 // Causal prefill attention on tcgen05 tensor cores (Sec. 5, "Chunked-Prefill
 // Stage", with the per-token sink + window rule for streaming heads).
 //
-// One CTA computes one 128-row query tile of one query head (rows are
-// consecutive positions). The KV tiles it visits come from a per-head
-// schedule: a retrieval head visits tiles 0 .. causal end; a streaming head
-// visits only the tiles holding its S sinks and the tiles that intersect the
-// W-token window of some row of the tile, so its cost is O(S + W) per row
-// instead of O(T). Tiles fully visible to every row skip the mask.
+// One CTA computes two consecutive 128-row query tiles (A = rows q0..q0+127,
+// B = rows q0+128..q0+255) of one query head against the same stream of
+// 128-key K/V tiles. The KV tiles visited come from a per-head schedule: a
+// retrieval head visits tiles 0 .. causal end; a streaming head only the
+// tiles holding its S sinks and the tiles that intersect the W-token window
+// of some row, so its cost is O(S + W) per row instead of O(T). Both query
+// tiles visit the union of their tile sets; a tile hidden from every row of
+// one query tile contributes zero weights there. Tiles fully visible to every
+// row of a query tile skip the mask.
 //
-// Warp roles (192 threads):
-//   warp 0      TMA producer: Q once, then K_j / V_j tiles into a 4-stage ring
-//               (4D tensor maps over [B][T][H][D], 128-byte swizzle).
-//   warp 1      TMEM owner and MMA issuer: S_j = Q K_j^T into one of two
-//               TMEM S buffers (so QK of tile j+1 overlaps softmax of tile j),
-//               then O += P_j V_j into the TMEM O accumulator.
-//   warps 2-5   softmax: thread r owns query row r (TMEM lane r). It reads
-//               its S row with tcgen05.ld, applies the mask, keeps the
-//               running max / sum in fp32 registers (the max only moves when
-//               it grows by more than 2^8, so O is rarely rescaled), writes
-//               P = exp2(S - m) as bf16 into shared memory in the swizzled
-//               K-major layout the MMA reads, and finally normalises O.
-// TMEM columns: S0 [0,128), S1 [128,256), O [256, 256 + D).
+// Warp roles (320 threads):
+//   warp 0      TMA producer: Q_A, Q_B once, then K_j / V_j tiles into a
+//               4-stage ring (4D tensor maps over [B][T][H][D], 128-byte swizzle).
+//   warp 1      TMEM owner and MMA issuer. S_X(j) = Q_X K_j^T reads both
+//               operands from shared memory; O_X += P_X(j) V_j reads P_X from
+//               TMEM, where the softmax wrote it over the first 64 columns of
+//               S_X. Per KV tile the issue order is O_A += P_A V, S_A(j+1),
+//               O_B += P_B V, S_B(j+1): a tile's next S overwrites its P only
+//               after the P.V that reads it (MMAs of one thread run in order),
+//               and while one query tile's softmax runs the tensor pipe works
+//               on the other's MMAs, hiding the commit -> softmax -> issue
+//               latency of each tile.
+//   warps 2-5   softmax of tile A, warps 6-9 softmax of tile B: thread r owns
+//               row r (TMEM lane r). One tcgen05.ld pass reads its S row, a
+//               two-range integer mask hides keys, max and sum reduce in 8
+//               independent chains, p = 2^(s*scale - m) costs one FFMA and one
+//               EX2, the running max moves only when it grows by more than
+//               2^8 (O rarely rescaled), and bf16 P pairs go back to TMEM with
+//               tcgen05.st (key k in column k/2, even k in the low half).
+// TMEM columns: S_A / P_A [0,128), S_B / P_B [128,256), O_A [256, 256+D),
+// O_B [256+D, 256+2D).
 #include <math.h>
 
 #include "common.cuh"
@@ -31,27 +42,28 @@ namespace aoh {
 namespace {
 
 using bf16 = __nv_bfloat16;
-constexpr int kBM = 128;  // query rows per tile
-constexpr int kBN = 128;  // keys per KV tile
-constexpr int kNS = 4;    // KV ring stages (K and V tiles alternate)
+constexpr int kBM = 128;         // rows per query tile (a CTA owns two)
+constexpr int kBN = 128;         // keys per KV tile
+constexpr int kNS = 4;           // KV ring stages (K and V tiles alternate)
 constexpr float kRescaleThreshold = 8.0f;
 constexpr uint32_t kTmemCols = 512;
+constexpr int kThreads = 320;
 
 template <int D>
 struct PfCfg {
   static constexpr int DBLK = D / 64;            // 64-wide column blocks (one TMA box each)
   static constexpr int BOX = 128 * 64 * 2;       // bytes of one [128 rows][64] box
-  static constexpr int QBYTES = DBLK * BOX;
+  static constexpr int QBYTES = DBLK * BOX;      // one query tile
   static constexpr int KVBYTES = DBLK * BOX;
-  static constexpr int PBYTES = 2 * BOX;         // one P buffer: [128 rows][128 keys]
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_KV = OFF_Q + QBYTES;
-  static constexpr int OFF_P = OFF_KV + kNS * KVBYTES;
-  static constexpr int OFF_BAR = OFF_P + 2 * PBYTES;
-  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 1 + 2 + 1;
+  static constexpr int OFF_Q = 0;                // Q_A, Q_B
+  static constexpr int OFF_KV = OFF_Q + 2 * QBYTES;
+  static constexpr int OFF_BAR = OFF_KV + kNS * KVBYTES;
+  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 2 + 2 + 1;
   static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;
   static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, false);
   static constexpr uint32_t IDESC_PV = idesc_bf16(kBM, D, true);
+  static_assert(SMEM <= 232448, "shared memory");
+  static_assert(256 + 2 * D <= (int)kTmemCols, "TMEM columns");
 };
 
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_t* err, volatile int* abort_flag) {
@@ -69,21 +81,20 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_
 }
 
 template <int D>
-__global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constant__ PrefillTcArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_constant__ PrefillTcArgs a) {
   using C = PfCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
   uint8_t* sQ = smem + C::OFF_Q;
   uint8_t* sKV = smem + C::OFF_KV;
-  uint8_t* sP = smem + C::OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* q_full = bars;
   uint64_t* kv_full = bars + 1;
   uint64_t* kv_empty = kv_full + kNS;
-  uint64_t* s_full = kv_empty + kNS;
-  uint64_t* s_empty = s_full + 2;
-  uint64_t* p_full = s_empty + 2;
-  uint64_t* pv_done = p_full + 1;  // [2]: PV of tile x completes pv_done[x & 1]
+  uint64_t* s_full = kv_empty + kNS;  // [2]: S_A, S_B ready
+  uint64_t* s_empty = s_full + 2;     // [2]: S_A, S_B read by the softmax
+  uint64_t* p_full = s_empty + 2;     // [2]: P_A, P_B written
+  uint64_t* pv_done = p_full + 2;     // [2]: O_A, O_B updated (P buffer free)
   uint64_t* drain = pv_done + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -95,8 +106,8 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
   const int kvh = h / g.G;
   const bool streaming = g.kind[kvh] != 0;
   const int len = a.lens[b];
-  const int q_end = min(q0 + kBM, len);
-  // KV tiles visited: [0, a_end) then [c_begin, c_end)
+  const int q_end = min(q0 + 2 * kBM, len);
+  // KV tiles visited (union of both query tiles): [0, a_end) then [c_begin, c_end)
   int a_end, c_begin, c_end;
   if (!streaming) {
     a_end = (q_end + kBN - 1) / kBN;
@@ -114,13 +125,12 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       mbar_init(&kv_full[s], 1);
       mbar_init(&kv_empty[s], 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&s_full[s], 1);
-      mbar_init(&s_empty[s], 4);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&s_full[x], 1);
+      mbar_init(&s_empty[x], 4);
+      mbar_init(&p_full[x], 4);
+      mbar_init(&pv_done[x], 1);
     }
-    mbar_init(p_full, 4);
-    mbar_init(&pv_done[0], 1);
-    mbar_init(&pv_done[1], 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -140,13 +150,15 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       prefetch_tmap(&a.tq);
       prefetch_tmap(&a.tk);
       prefetch_tmap(&a.tv);
-      mbar_arrive_expect_tx(q_full, C::QBYTES);
-      for (int db = 0; db < C::DBLK; ++db) tma_load_4d(sQ + db * C::BOX, &a.tq, db * 64, h, q0, b, q_full);
+      mbar_arrive_expect_tx(q_full, 2 * C::QBYTES);
+      for (int x = 0; x < 2; ++x)
+        for (int db = 0; db < C::DBLK; ++db)
+          tma_load_4d(sQ + x * C::QBYTES + db * C::BOX, &a.tq, db * 64, h, q0 + x * kBM, b, q_full);
       int issued = 0;
       for (int jj = 0; jj < n_tiles; ++jj) {
         const int j = jj < a_end ? jj : c_begin + (jj - a_end);
         bool ok = true;
-        for (int sel = 0; sel < 2 && ok; ++sel) {
+        for (int sel = 0; sel < 2; ++sel) {
           const int it = 2 * jj + sel;
           const int st = it % kNS;
           if (it >= kNS && !wait_bar(&kv_empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
@@ -169,59 +181,79 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t q_addr = smem_u32(sQ), kv_addr = smem_u32(sKV), p_addr = smem_u32(sP);
-      auto pv = [&](int x) -> bool {
-        const int it = 2 * x + 1, st = it % kNS;
-        if (!wait_bar(&kv_full[st], (it / kNS) & 1, a.err, abort_flag)) return false;
-        if (!wait_bar(p_full, x & 1, a.err, abort_flag)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = kv_addr + st * C::KVBYTES;
-        const uint32_t pb = p_addr + (x & 1) * C::PBYTES;
-#pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(pb + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc_sw128(v_addr + kk * 16 * 128, C::BOX, 1024);
-          tc_mma(tmem + 256, ad, bd, C::IDESC_PV, (x > 0 || kk > 0) ? 1u : 0u);
-        }
-        tc_commit(&pv_done[x & 1]);
-        tc_commit(&kv_empty[st]);
-        return true;
-      };
-      bool ok = wait_bar(q_full, 0, a.err, abort_flag);
-      tc_fence_after();
-      for (int jj = 0; jj < n_tiles && ok; ++jj) {
-        const int it = 2 * jj, st = it % kNS;
-        if (!wait_bar(&kv_full[st], (it / kNS) & 1, a.err, abort_flag)) { ok = false; break; }
-        if (jj >= 2 && !wait_bar(&s_empty[jj & 1], ((jj >> 1) & 1) ^ 1, a.err, abort_flag)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t k_addr = kv_addr + st * C::KVBYTES;
+      const uint32_t q_addr = smem_u32(sQ), kv_addr = smem_u32(sKV);
+      auto issue_s = [&](int x, int jj) {
+        const uint32_t k_addr = kv_addr + ((2 * jj) % kNS) * C::KVBYTES;
+        const uint32_t qa = q_addr + x * C::QBYTES;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(q_addr + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
+          const uint64_t ad = sdesc_sw128(qa + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
           const uint64_t bd = sdesc_sw128(k_addr + (kk >> 2) * C::BOX + (kk & 3) * 32, 16, 1024);
-          tc_mma(tmem + (jj & 1) * 128, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
+          tc_mma(tmem + x * 128, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&s_full[jj & 1]);
-        tc_commit(&kv_empty[st]);
-        if (jj >= 1 && !pv(jj - 1)) { ok = false; break; }
+        tc_commit(&s_full[x]);
+      };
+      auto issue_pv = [&](int x, int jj) {
+        const uint32_t v_addr = kv_addr + ((2 * jj + 1) % kNS) * C::KVBYTES;
+#pragma unroll
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          const uint64_t bd = sdesc_sw128(v_addr + kk * 16 * 128, C::BOX, 1024);
+          tc_mma_ts(tmem + 256 + x * D, tmem + x * 128 + kk * 8, bd, C::IDESC_PV, (jj > 0 || kk > 0) ? 1u : 0u);
+        }
+        tc_commit(&pv_done[x]);
+      };
+      auto wait_k = [&](int jj) { return wait_bar(&kv_full[(2 * jj) % kNS], ((2 * jj) / kNS) & 1, a.err, abort_flag); };
+      auto wait_v = [&](int jj) {
+        return wait_bar(&kv_full[(2 * jj + 1) % kNS], ((2 * jj + 1) / kNS) & 1, a.err, abort_flag);
+      };
+      bool ok = wait_bar(q_full, 0, a.err, abort_flag) && wait_k(0);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+        tc_commit(&kv_empty[0]);
       }
-      if (ok) pv(n_tiles - 1);
+      for (int jj = 0; jj < n_tiles && ok; ++jj) {
+        const bool more = jj + 1 < n_tiles;
+        const uint32_t ph = jj & 1;
+        // tile A: P_A(jj) sits in S_A's columns; S_A(jj+1) may overwrite them
+        // only after O_A += P_A(jj) V_jj is issued (same-thread MMAs run in order)
+        if (!wait_v(jj) || !wait_bar(&p_full[0], ph, a.err, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        issue_pv(0, jj);
+        if (more) {
+          if (!wait_k(jj + 1)) { ok = false; break; }
+          tc_fence_after();
+          issue_s(0, jj + 1);
+        }
+        if (!wait_bar(&p_full[1], ph, a.err, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        issue_pv(1, jj);
+        tc_commit(&kv_empty[(2 * jj + 1) % kNS]);
+        if (more) {
+          issue_s(1, jj + 1);
+          tc_commit(&kv_empty[(2 * (jj + 1)) % kNS]);
+        }
+      }
       tc_commit(drain);
       wait_bar(drain, 0, a.err, abort_flag);
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int q4 = warp & 3;
+    const int x = (warp - 2) >> 2;        // 0: tile A (warps 2-5), 1: tile B (warps 6-9)
+    const int q4 = warp & 3;              // TMEM lane quarter this warp may access
     const int r = q4 * 32 + lane;
-    const int i = q0 + r;
+    const int qx0 = q0 + x * kBM;         // first row of this query tile
+    const int i = qx0 + r;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+    const uint32_t s_col = x * 128, o_col = 256 + x * D;
     const int S = g.S, W = g.W;
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int jj = 0; jj < n_tiles; ++jj) {
       const int j = jj < a_end ? jj : c_begin + (jj - a_end);
       const int j0 = j * kBN;
-      if (!__all_sync(0xffffffffu, wait_bar(&s_full[jj & 1], (jj >> 1) & 1, a.err, abort_flag))) {
+      if (!__all_sync(0xffffffffu, wait_bar(&s_full[x], jj & 1, a.err, abort_flag))) {
         ok = false;
         break;
       }
@@ -229,11 +261,10 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       float s[kBN];
       {
         uint32_t v0[32], v1[32], v2[32], v3[32];
-        const uint32_t sb = tl + (jj & 1) * 128;
-        tmem_ld32(sb, v0);
-        tmem_ld32(sb + 32, v1);
-        tmem_ld32(sb + 64, v2);
-        tmem_ld32(sb + 96, v3);
+        tmem_ld32(tl + s_col, v0);
+        tmem_ld32(tl + s_col + 32, v1);
+        tmem_ld32(tl + s_col + 64, v2);
+        tmem_ld32(tl + s_col + 96, v3);
         tmem_ld_wait();
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
@@ -245,13 +276,13 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s_empty[jj & 1]);
+      if (lane == 0) mbar_arrive(&s_empty[x]);
 
       // hidden keys -> -inf. In tile coordinates key k is visible iff
       // k <= kmax (causal and inside the sequence) and, for a streaming head,
       // k < ks (a sink) or k >= kw (inside the window).
       const int jl = j0 + kBN - 1;
-      const bool full_vis = jl <= q0 && jl < len && (!streaming || jl < S || (q0 + kBM - 1) - j0 < W);
+      const bool full_vis = jl <= qx0 && jl < len && (!streaming || jl < S || (qx0 + kBM - 1) - j0 < W);
       if (!full_vis) {
         const int kmax = min(i, len - 1) - j0;
         const int ks = streaming ? S - j0 : kBN;
@@ -278,38 +309,31 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
       const bool warp_resc = __any_sync(0xffffffffu, resc) && jj > 0;
       const float neg_m = (m == -INFINITY) ? 0.f : -m;
 
-      // the P buffer of this tile was last read by PV of tile jj - 2
-      if (jj >= 2 && !__all_sync(0xffffffffu, wait_bar(&pv_done[jj & 1], ((jj - 2) >> 1) & 1, a.err, abort_flag))) {
-        ok = false;
-        break;
-      }
       // p = 2^(s * scale - m): one FFMA + one EX2 per element, hidden keys give
-      // 0; row sum in 8 chains; bf16 P straight into the swizzled K-major tile
-      uint8_t* prow = sP + (jj & 1) * C::PBYTES + r * 128;
+      // 0; row sum in 8 chains; bf16 pairs (key k in column k/2, even k low)
+      // written over the first 64 columns of this tile's S in TMEM
       float sum8[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) sum8[u] = 0.f;
 #pragma unroll
-      for (int ch = 0; ch < kBN / 8; ++ch) {
-        uint32_t w[4];
+      for (int hh = 0; hh < 4; ++hh) {
+        uint32_t w[16];
 #pragma unroll
-        for (int t = 0; t < 4; ++t) {
-          const int k = ch * 8 + 2 * t;
+        for (int t = 0; t < 16; ++t) {
+          const int k = hh * 32 + 2 * t;
           const float p0 = fast_exp2(fmaf(s[k], a.scale_log2, neg_m));
           const float p1 = fast_exp2(fmaf(s[k + 1], a.scale_log2, neg_m));
-          sum8[(ch * 4 + t) & 7] += p0 + p1;
+          sum8[t & 7] += p0 + p1;
           w[t] = float2_to_bf16x2(p0, p1);
         }
-        // key block ch / 8 (64 keys), 16-byte chunk ch % 8 of the 128-byte row
-        *reinterpret_cast<uint4*>(prow + (ch >> 3) * C::BOX + (((ch & 7) ^ (r & 7)) << 4)) =
-            make_uint4(w[0], w[1], w[2], w[3]);
+        tmem_st16(tl + s_col + hh * 16, w);
       }
       const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
       l = l * alpha + sum;
 
-      // rescale O (rare): PV of tile jj - 1 must have landed first
+      // rescale O (rare): O_X += P_X(jj-1) V must have landed first
       if (warp_resc) {
-        if (!__all_sync(0xffffffffu, wait_bar(&pv_done[(jj - 1) & 1], ((jj - 1) >> 1) & 1, a.err, abort_flag))) {
+        if (!__all_sync(0xffffffffu, wait_bar(&pv_done[x], (jj - 1) & 1, a.err, abort_flag))) {
           ok = false;
           break;
         }
@@ -317,28 +341,26 @@ __global__ void __launch_bounds__(192, 1) prefill_tc_kernel(const __grid_constan
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           uint32_t v[32];
-          tmem_ld32(tl + 256 + c * 32, v);
+          tmem_ld32(tl + o_col + c * 32, v);
           tmem_ld_wait();
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-          tmem_st32(tl + 256 + c * 32, v);
+          tmem_st32(tl + o_col + c * 32, v);
         }
-        tmem_st_wait();
       }
-      fence_proxy_async_smem();
+      tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_full);
+      if (lane == 0) mbar_arrive(&p_full[x]);
     }
-    if (ok && __all_sync(0xffffffffu,
-                         wait_bar(&pv_done[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1, a.err, abort_flag))) {
+    if (ok && __all_sync(0xffffffffu, wait_bar(&pv_done[x], (n_tiles - 1) & 1, a.err, abort_flag))) {
       tc_fence_after();
       const float inv = 1.f / l;
       bf16* op = static_cast<bf16*>(a.out) + (((size_t)b * a.T + min(i, len - 1)) * g.Hq + h) * D;
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t v[32];
-        tmem_ld32(tl + 256 + c * 32, v);
+        tmem_ld32(tl + o_col + c * 32, v);
         tmem_ld_wait();
         if (i < len) {
 #pragma unroll
@@ -397,7 +419,7 @@ cudaError_t launch_cfg(const PrefillTcArgs& a, int n_items, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  prefill_tc_kernel<D><<<n_items, 192, C::SMEM, s>>>(a);
+  prefill_tc_kernel<D><<<n_items, kThreads, C::SMEM, s>>>(a);
   return cudaGetLastError();
 }
 
