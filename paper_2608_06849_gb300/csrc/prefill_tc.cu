@@ -290,14 +290,17 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
 #pragma unroll
         for (int k = 0; k < kBN; ++k) s[k] = (k <= kmax && (k < ks || k >= kw)) ? s[k] : -INFINITY;
       }
-      // row max of the raw scores (the scale is positive) in 8 chains
+      // row max of the raw scores (the scale is positive): 8 chains of
+      // three-input max
       float mx8[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) mx8[u] = s[u];
+      for (int u = 0; u < 8; ++u) mx8[u] = fmaxf(s[u], s[u + 8]);
 #pragma unroll
-      for (int k = 8; k < kBN; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], s[k]);
-      const float rmax = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) *
+      for (int k = 16; k < kBN; k += 16)
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mx8[u] = fmax3f(mx8[u], s[k + u], s[k + 8 + u]);
+      const float rmax = fmax3f(fmax3f(mx8[0], mx8[1], mx8[2]), fmax3f(mx8[3], mx8[4], mx8[5]),
+                                fmaxf(mx8[6], mx8[7])) *
                          a.scale_log2;
       const float mn = fmaxf(m, rmax);
       const bool resc = mn > m + kRescaleThreshold;
@@ -309,26 +312,31 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
       const bool warp_resc = __any_sync(0xffffffffu, resc) && jj > 0;
       const float neg_m = (m == -INFINITY) ? 0.f : -m;
 
-      // p = 2^(s * scale - m): one FFMA + one EX2 per element, hidden keys give
-      // 0; row sum in 8 chains; bf16 pairs (key k in column k/2, even k low)
-      // written over the first 64 columns of this tile's S in TMEM
-      float sum8[8];
+      // p = 2^(s * scale - m), hidden keys give 0. Packed f32x2 arithmetic: one
+      // FFMA2 forms two exponent arguments and one FADD2 adds two weights into
+      // one of four pair accumulators. bf16 pairs (key k in column k/2, even k
+      // low) are written over the first 64 columns of this tile's S in TMEM.
+      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      const float2 nm2 = make_float2(neg_m, neg_m);
+      float2 sum4[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) sum8[u] = 0.f;
+      for (int u = 0; u < 4; ++u) sum4[u] = make_float2(0.f, 0.f);
 #pragma unroll
       for (int hh = 0; hh < 4; ++hh) {
         uint32_t w[16];
 #pragma unroll
         for (int t = 0; t < 16; ++t) {
           const int k = hh * 32 + 2 * t;
-          const float p0 = fast_exp2(fmaf(s[k], a.scale_log2, neg_m));
-          const float p1 = fast_exp2(fmaf(s[k + 1], a.scale_log2, neg_m));
-          sum8[t & 7] += p0 + p1;
-          w[t] = float2_to_bf16x2(p0, p1);
+          const float2 e = __ffma2_rn(make_float2(s[k], s[k + 1]), sc2, nm2);
+          const float2 pp = make_float2(fast_exp2(e.x), fast_exp2(e.y));
+          sum4[t & 3] = __fadd2_rn(sum4[t & 3], pp);
+          w[t] = float2_to_bf16x2(pp.x, pp.y);
         }
         tmem_st16(tl + s_col + hh * 16, w);
       }
-      const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+      const float2 s01 = __fadd2_rn(sum4[0], sum4[1]), s23 = __fadd2_rn(sum4[2], sum4[3]);
+      const float2 s03 = __fadd2_rn(s01, s23);
+      const float sum = s03.x + s03.y;
       l = l * alpha + sum;
 
       // rescale O (rare): O_X += P_X(jj-1) V must have landed first
