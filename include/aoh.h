@@ -51,7 +51,7 @@ typedef enum aoh_status {
   AOH_ERR_CUDA = 3,        /* a CUDA runtime call failed                           */
   AOH_ERR_TIMEOUT = 4,     /* a kernel's bounded wait ran out (see aoh_cache_check) */
   AOH_ERR_UNSUPPORTED = 5, /* d_head or group size outside the compiled kernels    */
-  AOH_ERR_STATE = 6        /* call not valid in the cache's current state          */
+  AOH_ERR_STATE = 6        /* reserved: call not valid in the cache's current state */
 } aoh_status;
 
 /* Labels of a KV head (one uint8 per KV head). */
@@ -105,18 +105,23 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
                           size_t kv_buffer_bytes, aoh_cache** out);
 
 /*
- * Causal prefill of an empty cache (the paper's prefill stage, Sec. 5 and the
- * inference-phase appendix; every streaming query uses the per-token
- * sink + window rule above).
+ * Causal prefill of one chunk of every sequence (Sec. 5, "Chunked-Prefill
+ * Stage"; every streaming query uses the per-token sink + window rule above).
+ * The chunk of sequence b holds positions L_b .. L_b + len_b - 1, where L_b
+ * is the number of tokens the cache already holds (0 for a first prefill):
+ * its rows attend to the cached prefix (retrieval heads: every earlier
+ * position; streaming heads: the sinks and the window, read from the sink and
+ * ring slots) and to the chunk itself. Its K/V are then appended (retrieval
+ * rows; streaming sinks and the last W positions of the new length).
  *   q    [B][T][n_q_heads][d_head]
  *   k, v [B][T][n_kv_heads][d_head]
- *   T    padded sequence length, 1 <= T <= max_seq.
- *   seq_lens  host array [B] of lengths 1..T, or NULL (all T). Rows at or
- *             past seq_lens[b] are not read and their outputs not written.
+ *   T    padded chunk length, >= 1.
+ *   seq_lens  host array [B] of chunk lengths 1..T, or NULL (all T). Rows at
+ *             or past seq_lens[b] are ignored: their contents (even NaN) do
+ *             not affect any output, and their outputs are not written.
  *   out  [B][T][n_q_heads][d_head], or NULL to only fill the cache.
- * Writes K/V of every position into the retrieval regions and the sinks plus
- * the last W positions into the streaming regions, then sets the lengths.
- * Errors: INVALID, CAPACITY (T > max_seq), STATE (cache not empty), CUDA.
+ * Errors: INVALID, CAPACITY (a retrieval head would pass max_seq; nothing is
+ * launched), CUDA.
  */
 aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T,
                        const int32_t* seq_lens, aoh_cache* cache, void* out, void* stream);

@@ -64,24 +64,28 @@ aoh_status check_config(const aoh_config* cfg, const uint8_t* labels, int* n_r, 
 // Prefill work: one item per (b, query head, 128-row query tile), with the
 // number of 128-key tiles it visits as its cost; heaviest first so the
 // hardware block scheduler fills the machine longest-processing-time first.
-std::vector<int4> prefill_schedule(const CacheGeom& g, const std::vector<int32_t>& lens) {
+std::vector<int4> prefill_schedule(const CacheGeom& g, const std::vector<int32_t>& base,
+                                   const std::vector<int32_t>& lens) {
   constexpr int BM = 256, BN = 128;
   std::vector<int4> items;
   for (int b = 0; b < g.B; ++b) {
     for (int h = 0; h < g.Hq; ++h) {
       const bool streaming = g.kind[h / g.G] != 0;
+      const int Lb = base[b];
+      const int n_c = Lb == 0 ? 0 : ((streaming ? std::min(Lb, g.S + g.W) : Lb) + BN - 1) / BN;
+      const int S_rel = g.S - Lb;
       for (int q0 = 0; q0 < lens[b]; q0 += BM) {
         const int q_end = std::min(q0 + BM, (int)lens[b]);
         int n;
         if (!streaming) {
           n = (q_end + BN - 1) / BN;
         } else {
-          const int a_end = (std::min(g.S, q_end) + BN - 1) / BN;
+          const int a_end = (std::min(std::max(S_rel, 0), q_end) + BN - 1) / BN;
           const int c_begin = std::max(a_end, std::max(0, q0 - g.W + 1) / BN);
           const int c_end = std::max(c_begin, (q_end + BN - 1) / BN);
           n = a_end + (c_end - c_begin);
         }
-        items.push_back(make_int4(b, h, q0, n));
+        items.push_back(make_int4(b, h, q0, n_c + n));
       }
     }
   }
@@ -110,6 +114,7 @@ struct aoh_cache {
   // device metadata (one allocation)
   void* meta = nullptr;
   int32_t* d_lens = nullptr;
+  int32_t* d_chunk = nullptr;  // rows of the current prefill chunk
   uint32_t* d_counters = nullptr;
   uint32_t* d_done = nullptr;
   uint32_t* d_err = nullptr;
@@ -186,7 +191,7 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   const size_t n_lens = ((size_t)c.batch + 63) / 64 * 64;
   const size_t n_cnt = ((size_t)c.batch * c.n_kv_heads + 63) / 64 * 64;
   const size_t n_part = decode_partial_floats(2 * h->num_sms, G, c.d_head);
-  const size_t meta_bytes = (n_lens + n_cnt + 64) * 4 + n_part * 4;
+  const size_t meta_bytes = (2 * n_lens + n_cnt + 64) * 4 + n_part * 4;
   e = cudaMalloc(&h->meta, meta_bytes);
   if (e == cudaSuccess) e = cudaMemset(h->meta, 0, meta_bytes);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -197,10 +202,11 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   }
   uint32_t* base = static_cast<uint32_t*>(h->meta);
   h->d_lens = reinterpret_cast<int32_t*>(base);
-  h->d_counters = base + n_lens;
+  h->d_chunk = reinterpret_cast<int32_t*>(base + n_lens);
+  h->d_counters = base + 2 * n_lens;
   h->d_done = h->d_counters + n_cnt;
   h->d_err = h->d_done + 32;
-  h->d_partials = reinterpret_cast<float*>(base + n_lens + n_cnt + 64);
+  h->d_partials = reinterpret_cast<float*>(base + 2 * n_lens + n_cnt + 64);
   *out = h;
   return AOH_OK;
 }
@@ -262,60 +268,72 @@ aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, c
     return fail(AOH_ERR_INVALID, "q, k, v and out must be 16-byte aligned");
   const CacheGeom& g = cache->geom;
   if (T < 1) return fail(AOH_ERR_INVALID, "T must be >= 1");
-  if (T > g.max_seq) return fail(AOH_ERR_CAPACITY, "T = %d exceeds max_seq = %d", T, g.max_seq);
-  for (int b = 0; b < g.B; ++b)
-    if (cache->lens[b] != 0) return fail(AOH_ERR_STATE, "prefill needs an empty cache (sequence %d holds %d tokens)", b, cache->lens[b]);
-  std::vector<int32_t> lens(g.B, T);
+  std::vector<int32_t> clen(g.B, T);
   if (seq_lens) {
     for (int b = 0; b < g.B; ++b) {
       if (seq_lens[b] < 1 || seq_lens[b] > T)
         return fail(AOH_ERR_INVALID, "seq_lens[%d] = %d is outside [1, T]", b, seq_lens[b]);
-      lens[b] = seq_lens[b];
+      clen[b] = seq_lens[b];
     }
   }
+  const std::vector<int32_t> base = cache->lens;
+  std::vector<int32_t> lens(g.B);
+  bool chunked = false;
+  for (int b = 0; b < g.B; ++b) {
+    lens[b] = base[b] + clen[b];
+    chunked |= base[b] > 0;
+    if (g.n_r > 0 && lens[b] > g.max_seq)
+      return fail(AOH_ERR_CAPACITY, "sequence %d would hold %d tokens; max_seq is %d", b, lens[b], g.max_seq);
+  }
   cudaStream_t s = (cudaStream_t)stream;
-  cudaError_t e = cudaMemcpyAsync(cache->d_lens, lens.data(), sizeof(int32_t) * g.B, cudaMemcpyHostToDevice, s);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(lens)");
+  cudaError_t e = cudaMemcpyAsync(cache->d_chunk, clen.data(), sizeof(int32_t) * g.B, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(chunk lengths)");
+
+  // attention first: a chunk's own writes to a streaming ring would overwrite
+  // positions its rows still read
+  if (out) {
+    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
+    std::vector<int4> items = prefill_schedule(g, base, clen);
+    if (items.size() > cache->work_cap) {
+      if (cache->d_work) cudaFree(cache->d_work);
+      cache->d_work = nullptr;
+      cache->work_cap = 0;
+      e = cudaMalloc(&cache->d_work, items.size() * sizeof(int4));
+      if (e != cudaSuccess) return cuda_fail(e, "work list allocation");
+      cache->work_cap = items.size();
+    }
+    e = cudaMemcpyAsync(cache->d_work, items.data(), items.size() * sizeof(int4), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work)");
+    PrefillTcArgs pa;
+    memset(&pa, 0, sizeof(pa));
+    pa.geom = g;
+    pa.out = out;
+    pa.lens = cache->d_chunk;
+    pa.base = cache->d_lens;
+    pa.work = cache->d_work;
+    pa.err = cache->d_err;
+    pa.T = T;
+    pa.scale_log2 = scale_log2;
+    if (!prefill_tc_make_maps(&pa, q, k, v, g.B, T))
+      return fail(AOH_ERR_CUDA, "cuTensorMapEncodeTiled failed for q/k/v");
+    if (chunked && !prefill_tc_make_cache_maps(&pa, cache->kv))
+      return fail(AOH_ERR_CUDA, "cuTensorMapEncodeTiled failed for the cache");
+    e = launch_prefill_tc(pa, (int)items.size(), s);
+    if (e != cudaSuccess) return cuda_fail(e, "prefill kernel launch");
+  }
 
   AppendArgs ap;
   ap.geom = g;
   ap.k = k;
   ap.v = v;
   ap.kv = cache->kv;
-  ap.lens = cache->d_lens;
+  ap.lens = cache->d_chunk;
+  ap.base = cache->d_lens;
   ap.T = T;
   e = launch_append(ap, s);
   if (e != cudaSuccess) return cuda_fail(e, "append kernel launch");
-
-  if (out) {
-    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
-    {
-      std::vector<int4> items = prefill_schedule(g, lens);
-      if (items.size() > cache->work_cap) {
-        if (cache->d_work) cudaFree(cache->d_work);
-        cache->d_work = nullptr;
-        cache->work_cap = 0;
-        e = cudaMalloc(&cache->d_work, items.size() * sizeof(int4));
-        if (e != cudaSuccess) return cuda_fail(e, "work list allocation");
-        cache->work_cap = items.size();
-      }
-      e = cudaMemcpyAsync(cache->d_work, items.data(), items.size() * sizeof(int4), cudaMemcpyHostToDevice, s);
-      if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work)");
-      PrefillTcArgs pa;
-      memset(&pa, 0, sizeof(pa));
-      pa.geom = g;
-      pa.out = out;
-      pa.lens = cache->d_lens;
-      pa.work = cache->d_work;
-      pa.err = cache->d_err;
-      pa.T = T;
-      pa.scale_log2 = scale_log2;
-      if (!prefill_tc_make_maps(&pa, q, k, v, g.B, T))
-        return fail(AOH_ERR_CUDA, "cuTensorMapEncodeTiled failed for q/k/v");
-      e = launch_prefill_tc(pa, (int)items.size(), s);
-      if (e != cudaSuccess) return cuda_fail(e, "prefill kernel launch");
-    }
-  }
+  e = launch_lens_add(cache->d_lens, cache->d_chunk, g.B, s);
+  if (e != cudaSuccess) return cuda_fail(e, "length update launch");
   cache->lens = lens;
   return AOH_OK;
 }

@@ -56,7 +56,8 @@ struct AppendArgs {
   const void* k;  // [B][T][Hkv][D]
   const void* v;
   void* kv;
-  const int32_t* lens;  // device [B]
+  const int32_t* lens;  // device [B]: rows of the chunk
+  const int32_t* base;  // device [B]: tokens cached before the chunk
   int T;
 };
 
@@ -64,10 +65,12 @@ struct AppendArgs {
 // ([B][T][H][D], box 128 rows x 64 columns, 128-byte swizzle) and a work list
 // of (b, query head, first row) tiles sorted by cost.
 struct alignas(64) PrefillTcArgs {
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv;  // the chunk's q / k / v
+  CUtensorMap tcr, tcs;    // cache: retrieval / streaming regions as [regions][K, V][rows][D]
   CacheGeom geom;
   void* out;            // [B][T][Hq][D]
-  const int32_t* lens;  // device [B]
+  const int32_t* lens;  // device [B]: rows of the chunk
+  const int32_t* base;  // device [B]: tokens cached before the chunk
   const int4* work;     // {b, h, q0, cost}
   uint32_t* err;
   int T;
@@ -79,6 +82,7 @@ void record_error(const char* msg);
 
 // Launchers (return the launch's cudaError_t).
 bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const void* v, int B, int T);
+bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
 // CTAs for a decode launch over `total_rows` cached rows on `num_sms` SMs.
@@ -86,6 +90,7 @@ int decode_ctas(long long total_rows, int num_sms);
 // Floats of the partial buffer for `n_ctas` CTAs.
 size_t decode_partial_floats(int n_ctas, int G, int D);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
+cudaError_t launch_lens_add(int32_t* lens, const int32_t* add, int B, cudaStream_t s);
 bool decode_supported(int D, int G);
 
 }  // namespace aoh

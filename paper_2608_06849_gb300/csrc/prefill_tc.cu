@@ -1,5 +1,10 @@
 // Causal prefill attention on tcgen05 tensor cores (Sec. 5, "Chunked-Prefill
-// Stage", with the per-token sink + window rule for streaming heads).
+// Stage", with the per-token sink + window rule for streaming heads). A call
+// processes one chunk of every sequence: rows at positions Lb .. Lb + len - 1
+// after Lb cached tokens (Lb = 0 for a first prefill). Cached keys are read
+// from the KV cache itself (retrieval rows, or the streaming sink + ring
+// slots) before the chunk's own keys; the cache is appended after this
+// kernel, so the ring still holds the positions the chunk's rows need.
 //
 // One CTA computes two consecutive 128-row query tiles (A = rows q0..q0+127,
 // B = rows q0+128..q0+255) of one query head against the same stream of
@@ -58,7 +63,7 @@ struct PfCfg {
   static constexpr int OFF_Q = 0;                // Q_A, Q_B
   static constexpr int OFF_KV = OFF_Q + 2 * QBYTES;
   static constexpr int OFF_BAR = OFF_KV + kNS * KVBYTES;
-  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 2 + 2 + 1;
+  static constexpr int NBAR = 1 + 2 * kNS + 2 + 2 + 2 + 2 + 1 + 2;
   static constexpr int SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;
   static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, false);
   static constexpr uint32_t IDESC_PV = idesc_bf16(kBM, D, true);
@@ -80,6 +85,15 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_
   }
 }
 
+// Bits lo..hi-1 of a 32-bit word (lo, hi clamped to [0, 32]).
+__device__ __forceinline__ uint32_t range_bits(int lo, int hi) {
+  lo = max(lo, 0);
+  hi = min(hi, 32);
+  if (hi <= lo) return 0u;
+  const uint32_t top = hi == 32 ? 0xffffffffu : ((1u << hi) - 1u);
+  return top & ~((1u << lo) - 1u);
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_constant__ PrefillTcArgs a) {
   using C = PfCfg<D>;
@@ -96,7 +110,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
   uint64_t* p_full = s_empty + 2;     // [2]: P_A, P_B written
   uint64_t* pv_done = p_full + 2;     // [2]: O_A, O_B updated (P buffer free)
   uint64_t* drain = pv_done + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  // [2]: padding rows of the item's first / second partial V tile are zeroed.
+  // Only the last cache tile and the chunk tile holding row len - 1 can be
+  // partial, so each barrier completes at most once per item.
+  uint64_t* v_zeroed = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(v_zeroed + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -106,18 +124,28 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
   const int kvh = h / g.G;
   const bool streaming = g.kind[kvh] != 0;
   const int len = a.lens[b];
+  const int Lb = a.base[b];
   const int q_end = min(q0 + 2 * kBM, len);
+  const int S_rel = g.S - Lb;
+  const int n_c = Lb == 0 ? 0 : ((streaming ? min(Lb, g.S + g.W) : Lb) + kBN - 1) / kBN;
   // KV tiles visited (union of both query tiles): [0, a_end) then [c_begin, c_end)
   int a_end, c_begin, c_end;
   if (!streaming) {
     a_end = (q_end + kBN - 1) / kBN;
     c_begin = c_end = a_end;
   } else {
-    a_end = (min(g.S, q_end) + kBN - 1) / kBN;
+    a_end = (min(max(S_rel, 0), q_end) + kBN - 1) / kBN;
     c_begin = max(a_end, max(0, q0 - g.W + 1) / kBN);
     c_end = max(c_begin, (q_end + kBN - 1) / kBN);
   }
-  const int n_tiles = a_end + (c_end - c_begin);
+  const int n_tiles = n_c + a_end + (c_end - c_begin);
+  // keys of KV tile jj that hold data (the rest: cache rows not yet written,
+  // or chunk padding); fewer than kBN makes the tile partial
+  auto tile_valid = [&](int jj) {
+    if (jj < n_c) return (streaming ? min(Lb, g.S + g.W) : Lb) - jj * kBN;
+    const int jc = jj - n_c;
+    return len - (jc < a_end ? jc : c_begin + (jc - a_end)) * kBN;
+  };
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -132,6 +160,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
       mbar_init(&pv_done[x], 1);
     }
     mbar_init(drain, 1);
+    mbar_init(&v_zeroed[0], 1);
+    mbar_init(&v_zeroed[1], 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -146,6 +176,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
+    // Lane 0 issues the copies. Rows of a V tile past its valid keys may hold
+    // anything (cache rows not yet written, chunk padding) and a zero weight
+    // times a NaN is still NaN, so for a partial V tile the whole warp waits
+    // for the copy, zeroes those rows and signals v_zeroed before the MMA
+    // issuer may read the tile.
     if (lane == 0) {
       prefetch_tmap(&a.tq);
       prefetch_tmap(&a.tk);
@@ -154,30 +189,64 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
       for (int x = 0; x < 2; ++x)
         for (int db = 0; db < C::DBLK; ++db)
           tma_load_4d(sQ + x * C::QBYTES + db * C::BOX, &a.tq, db * 64, h, q0 + x * kBM, b, q_full);
-      int issued = 0;
-      for (int jj = 0; jj < n_tiles; ++jj) {
-        const int j = jj < a_end ? jj : c_begin + (jj - a_end);
-        bool ok = true;
-        for (int sel = 0; sel < 2; ++sel) {
-          const int it = 2 * jj + sel;
-          const int st = it % kNS;
+    }
+    int issued = 0, n_partial = 0;
+    bool ok = true;
+    for (int jj = 0; jj < n_tiles && ok; ++jj) {
+      const int jc = jj - n_c;
+      const int j = jc < a_end ? jc : c_begin + (jc - a_end);
+      for (int sel = 0; sel < 2; ++sel) {
+        const int it = 2 * jj + sel;
+        const int st = it % kNS;
+        if (lane == 0) {
           if (it >= kNS && !wait_bar(&kv_empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
+            ok = false;
+          } else {
+            mbar_arrive_expect_tx(&kv_full[st], C::KVBYTES);
+            if (jj < n_c) {
+              // cache region viewed as [regions][K, V][rows][D]
+              const CUtensorMap* map = streaming ? &a.tcs : &a.tcr;
+              const int region = streaming ? b * g.n_s + g.idx[kvh] : b * g.n_r + g.idx[kvh];
+              for (int db = 0; db < C::DBLK; ++db)
+                tma_load_4d(sKV + st * C::KVBYTES + db * C::BOX, map, db * 64, jj * kBN, sel, region,
+                            &kv_full[st]);
+            } else {
+              const CUtensorMap* map = sel ? &a.tv : &a.tk;
+              for (int db = 0; db < C::DBLK; ++db)
+                tma_load_4d(sKV + st * C::KVBYTES + db * C::BOX, map, db * 64, kvh, j * kBN, b, &kv_full[st]);
+            }
+            issued = it + 1;
+          }
+        }
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        const int valid = tile_valid(jj);
+        if (sel == 1 && valid < kBN && n_partial < 2) {
+          if (!__all_sync(0xffffffffu, wait_bar(&kv_full[st], (it / kNS) & 1, a.err, abort_flag))) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&kv_full[st], C::KVBYTES);
-          const CUtensorMap* map = sel ? &a.tv : &a.tk;
-          for (int db = 0; db < C::DBLK; ++db)
-            tma_load_4d(sKV + st * C::KVBYTES + db * C::BOX, map, db * 64, kvh, j * kBN, b, &kv_full[st]);
-          issued = it + 1;
+          uint8_t* vt = sKV + st * C::KVBYTES;
+          for (int idx = max(valid, 0) * 8 + lane; idx < kBN * 8; idx += 32) {  // 16-byte chunks
+            const int row = idx >> 3, chunk = idx & 7;
+#pragma unroll
+            for (int db = 0; db < C::DBLK; ++db)
+              *reinterpret_cast<uint4*>(vt + db * C::BOX + row * 128 + chunk * 16) = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&v_zeroed[n_partial]);
+          ++n_partial;
         }
-        if (!ok) break;
       }
-      // every issued copy lands before the CTA can exit
+    }
+    // every issued copy lands before the CTA can exit
+    if (lane == 0) {
       wait_bar(q_full, 0, a.err, abort_flag);
       for (int it = issued > kNS ? issued - kNS : 0; it < issued; ++it)
         wait_bar(&kv_full[it % kNS], (it / kNS) & 1, a.err, abort_flag);
     }
+    __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -203,8 +272,14 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
         tc_commit(&pv_done[x]);
       };
       auto wait_k = [&](int jj) { return wait_bar(&kv_full[(2 * jj) % kNS], ((2 * jj) / kNS) & 1, a.err, abort_flag); };
+      int n_partial = 0;  // partial V tiles seen so far (index into v_zeroed)
       auto wait_v = [&](int jj) {
-        return wait_bar(&kv_full[(2 * jj + 1) % kNS], ((2 * jj + 1) / kNS) & 1, a.err, abort_flag);
+        if (!wait_bar(&kv_full[(2 * jj + 1) % kNS], ((2 * jj + 1) / kNS) & 1, a.err, abort_flag)) return false;
+        if (tile_valid(jj) < kBN && n_partial < 2) {
+          if (!wait_bar(&v_zeroed[n_partial], 0, a.err, abort_flag)) return false;
+          ++n_partial;
+        }
+        return true;
       };
       bool ok = wait_bar(q_full, 0, a.err, abort_flag) && wait_k(0);
       if (ok) {
@@ -248,10 +323,12 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     const uint32_t s_col = x * 128, o_col = 256 + x * D;
     const int S = g.S, W = g.W;
+    const int rot = (streaming && Lb > S + W) ? (Lb - S) % W : 0;
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int jj = 0; jj < n_tiles; ++jj) {
-      const int j = jj < a_end ? jj : c_begin + (jj - a_end);
+      const int jc = jj - n_c;
+      const int j = jj < n_c ? jj : (jc < a_end ? jc : c_begin + (jc - a_end));
       const int j0 = j * kBN;
       if (!__all_sync(0xffffffffu, wait_bar(&s_full[x], jj & 1, a.err, abort_flag))) {
         ok = false;
@@ -281,14 +358,55 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
       // hidden keys -> -inf. In tile coordinates key k is visible iff
       // k <= kmax (causal and inside the sequence) and, for a streaming head,
       // k < ks (a sink) or k >= kw (inside the window).
-      const int jl = j0 + kBN - 1;
-      const bool full_vis = jl <= qx0 && jl < len && (!streaming || jl < S || (qx0 + kBM - 1) - j0 < W);
-      if (!full_vis) {
+      // Hidden keys -> -inf. Every tile kind reduces to visible key ranges
+      // [e_lo, e_hi), [a0, a1), [b0, b1) in tile coordinates, turned into four
+      // 32-bit masks (one per 32 keys) so that each score costs one AND with
+      // an immediate and one select.
+      bool need_mask;
+      int e_hi = kBN, a0 = 0, a1 = 0, b0 = 0, b1 = 0;
+      if (jj < n_c) {
+        if (!streaming) {
+          need_mask = j0 + kBN > Lb;
+          e_hi = Lb - j0;
+        } else {
+          need_mask = true;
+          e_hi = min(S, Lb) - j0;
+          if (Lb <= S + W) {
+            a0 = max(S, Lb + i - W + 1) - j0;
+            a1 = Lb - j0;
+          } else if (i + 1 < W) {
+            const int u = rot + i + 1;
+            if (u < W) {
+              a0 = S + u - j0;
+              a1 = S + W - j0;
+              b0 = S - j0;
+              b1 = S + rot - j0;
+            } else {
+              a0 = S + u - W - j0;
+              a1 = S + rot - j0;
+            }
+          }
+        }
+      } else {
+        const int jl = j0 + kBN - 1;
+        need_mask = !(jl <= qx0 && jl < len && (!streaming || jl < S_rel || (qx0 + kBM - 1) - j0 < W));
         const int kmax = min(i, len - 1) - j0;
-        const int ks = streaming ? S - j0 : kBN;
-        const int kw = streaming ? i - W + 1 - j0 : 0;
+        if (!streaming) {
+          e_hi = kmax + 1;
+        } else {
+          e_hi = min(kmax + 1, S_rel - j0);
+          a0 = i - W + 1 - j0;
+          a1 = kmax + 1;
+        }
+      }
+      if (need_mask) {
 #pragma unroll
-        for (int k = 0; k < kBN; ++k) s[k] = (k <= kmax && (k < ks || k >= kw)) ? s[k] : -INFINITY;
+        for (int c = 0; c < 4; ++c) {
+          const uint32_t vm = range_bits(0, e_hi - 32 * c) | range_bits(a0 - 32 * c, a1 - 32 * c) |
+                              range_bits(b0 - 32 * c, b1 - 32 * c);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) s[32 * c + e] = (vm & (1u << e)) ? s[32 * c + e] : -INFINITY;
+        }
       }
       // row max of the raw scores (the scale is positive): 8 chains of
       // three-input max
@@ -437,6 +555,30 @@ bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const 
   const CacheGeom& g = a->geom;
   return make_map(&a->tq, q, B, T, g.Hq, g.D) && make_map(&a->tk, k, B, T, g.Hkv, g.D) &&
          make_map(&a->tv, v, B, T, g.Hkv, g.D);
+}
+
+// 4D map over one kind of cache region: [regions][K, V][cap rows][D], box
+// [1][1][128][64], 128-byte swizzle. Rows past `cap` read as zeros.
+static bool make_region_map(CUtensorMap* map, const void* base, int regions, int cap, int D) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)cap, 2, (cuuint64_t)regions};
+  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)cap * D * 2, (cuuint64_t)cap * D * 2 * 2};
+  cuuint32_t box[4] = {64, 128, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv) {
+  const CacheGeom& g = a->geom;
+  const bf16* base = static_cast<const bf16*>(kv);
+  bool ok = true;
+  if (g.n_r > 0) ok = ok && make_region_map(&a->tcr, base + g.r_region(0, 0), g.B * g.n_r, g.max_seq, g.D);
+  if (g.n_s > 0) ok = ok && make_region_map(&a->tcs, base + g.s_region(0, 0), g.B * g.n_s, g.S + g.W, g.D);
+  return ok;
 }
 
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s) {

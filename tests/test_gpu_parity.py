@@ -73,9 +73,9 @@ def test_decode_past_capacity_is_refused():
     with pytest.raises(aoh.AohError) as e:
         cache.decode_step(q1, k1, k1, torch.empty_like(q1))
     assert e.value.status == 2
-    with pytest.raises(aoh.AohError) as e:
+    with pytest.raises(aoh.AohError) as e:            # a further chunk would pass max_seq
         cache.prefill(k.repeat(1, 1, 4, 1), k, k)
-    assert e.value.status == 6
+    assert e.value.status == 2
     cache.reset()
     cache.prefill(k.repeat(1, 1, 4, 1), k, k)
     assert cache.lens() == [4]
