@@ -299,6 +299,32 @@ def run_native(args):
     pre_tflops_total = ranks.sum(flops) / (pre_ms * 1e-3) / 1e12
     pcache.close()
 
+    # ---------------- chunked prefill leg: the same 32K prefill in chunks
+    n_chunks = args.prefill_chunks
+    C = T // n_chunks
+    chunks = [(q[:, i * C:(i + 1) * C].contiguous(), k[:, i * C:(i + 1) * C].contiguous(),
+               v[:, i * C:(i + 1) * C].contiguous()) for i in range(n_chunks)]
+    couts = [torch.empty_like(ch[0]) for ch in chunks]
+    ccache = aoh.Cache(1, pwl.n_q_heads, pwl.n_kv_heads, pwl.d_head, T, pwl.sink, pwl.window, plabels)
+    for _ in range(max(W, 3)):
+        ccache.reset()
+        for ch, co in zip(chunks, couts):
+            ccache.prefill(ch[0], ch[1], ch[2], co)
+    ccache.check()
+    cev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    barrier()
+    cev[0].record(stream)
+    for _ in range(Kp):
+        ccache.reset()
+        for ch, co in zip(chunks, couts):
+            ccache.prefill(ch[0], ch[1], ch[2], co)
+    cev[1].record(stream)
+    barrier()
+    chunk_ms = max_over_ranks(cev[0].elapsed_time(cev[1])) / Kp
+    ccache.check()
+    ccache.close()
+    del chunks, couts
+
     # ---------------- cpu baseline (oracle on a bounded sample), rank 0 only
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -341,6 +367,9 @@ def run_native(args):
                                  "unit": "TFLOP/s", "frac": round(pre_tflops / tf_peak, 4),
                                  "traffic": traffic_for("prefill"),
                                  "peak_note": f"{peak_note} dense bf16 (burst); time includes the cache append"}},
+        "chunked_prefill": {"chunks": n_chunks, "chunk_tokens": C, "ms": round(chunk_ms, 3),
+                            "tflops": round(flops / (chunk_ms * 1e-3) / 1e12, 2),
+                            "note": "same 32K prefill as consecutive chunks; each chunk reads the cached prefix"},
         "e2e": {"value": round(e2e_us, 3), "unit": "us/step", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": K,
         "clocks": clock_info,
@@ -444,6 +473,121 @@ def run_reference(args):
     print(json.dumps(line))
 
 
+# ------------------------------------------------------- other workloads
+
+def _decode_timing(aoh, torch, cache, wl, steps, warmup):
+    from paper_2608_06849_gb300.workloads import decode_inputs
+    inputs = [decode_inputs(wl, s, device="cuda") for s in range(warmup + steps)]
+    out = torch.empty(wl.batch, wl.n_q_heads, wl.d_head, dtype=torch.bfloat16, device="cuda")
+    for s in range(warmup):
+        cache.decode_step(*inputs[s], out)
+    cache.check()
+    before = cache.lens()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for s in range(steps):
+        cache.decode_step(*inputs[warmup + s], out)
+    e1.record()
+    torch.cuda.synchronize()
+    cache.check()
+    return e0.elapsed_time(e1) * 1000.0 / steps, before
+
+
+def run_ragged(args):
+    """Decode of 64 sequences with lengths uniform in [4K, 32K], S = 64:
+    streaming fraction x window sweep (one JSON line, one entry per point)."""
+    import dataclasses
+
+    import torch
+
+    from paper_2608_06849_gb300 import aoh
+    from paper_2608_06849_gb300 import build as aoh_build
+    from paper_2608_06849_gb300.workloads import RAGGED, labels_for, randn_bf16, seq_lens
+    aoh_build.build()
+    aoh.load()
+    peaks, note = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    lens = seq_lens(RAGGED)
+    T = max(lens)
+    B, Hkv, D = RAGGED.batch, RAGGED.n_kv_heads, RAGGED.d_head
+    kfill = randn_bf16((B, T, Hkv, D), 7101, "cuda")
+    vfill = randn_bf16((B, T, Hkv, D), 7102, "cuda")
+    points = []
+    for frac in (0.0, 0.25, 0.5, 0.75):
+        for W in (512, 2048, 8192):
+            wl = dataclasses.replace(RAGGED, n_streaming=int(frac * Hkv), window=W)
+            labels = labels_for(wl)
+            cache = aoh.Cache(B, wl.n_q_heads, Hkv, D, T + args.steps + args.warmup + 4, wl.sink, W, labels)
+            cache.prefill(None, kfill, vfill, None, seq_lens=lens)
+            us, before = _decode_timing(aoh, torch, cache, wl, args.steps, args.warmup)
+            nbytes = decode_bytes(before, labels, wl)
+            points.append({"streaming_frac": frac, "window": W, "us_per_step": round(us, 2),
+                           "bytes_per_step": nbytes, "hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
+                           "frac_of_peak": round(nbytes / (us * 1e-6) / 1e9 / hbm, 4)})
+            cache.close()
+    print(json.dumps({"workload": f"{RAGGED.name}: B={B} Hq={RAGGED.n_q_heads} Hkv={Hkv} d={D} "
+                                  f"lens uniform [4096, 32768] seed {RAGGED.seed} S={RAGGED.sink}",
+                      "metric": "decode attn us/step and HBM GB/s", "steps": args.steps, "warmup": args.warmup,
+                      "peak_hbm_gbs": hbm, "peak_note": note, "sweep": points}))
+
+
+def run_stack(args):
+    """One layer of the 28-layer Qwen2.5-7B-shaped stack at 256K: per-layer
+    prefill latency and decode latency, and the whole stack's KV bytes
+    against the all-retrieval layout."""
+    import torch
+
+    from paper_2608_06849_gb300 import aoh
+    from paper_2608_06849_gb300 import build as aoh_build
+    from paper_2608_06849_gb300.workloads import STACK_256K, labels_for, prefill_inputs
+    aoh_build.build()
+    aoh.load()
+    peaks, note = load_peaks()
+    wl = STACK_256K
+    T = wl.prefill_len
+    labels = labels_for(wl, layer=0)
+    q, k, v = prefill_inputs(wl, device="cuda")
+    cache = aoh.Cache(1, wl.n_q_heads, wl.n_kv_heads, wl.d_head, T + args.steps + args.warmup + 4, wl.sink,
+                      wl.window, labels)
+    out = torch.empty_like(q)
+    for _ in range(2):
+        cache.reset()
+        cache.prefill(q, k, v, out)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 3
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        cache.reset()
+        cache.prefill(q, k, v, out)
+    e1.record()
+    torch.cuda.synchronize()
+    cache.check()
+    pre_ms = e0.elapsed_time(e1) / reps
+    flops = prefill_flops(wl, labels, T)
+    del q, out
+    us, before = _decode_timing(aoh, torch, cache, wl, args.steps, args.warmup)
+    nbytes = decode_bytes(before, labels, wl)
+    cfg = cache.cfg
+    kv_aoh = sum(aoh.aoh_cache_bytes(cfg, labels_for(wl, layer=L)) for L in range(wl.layers))
+    kv_full = wl.layers * aoh.aoh_cache_bytes(cfg, [0] * wl.n_kv_heads)
+    cache.close()
+    tf_peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    print(json.dumps({
+        "workload": f"{wl.name}: {wl.layers} layers x (Hq={wl.n_q_heads} Hkv={wl.n_kv_heads} d={wl.d_head}), "
+                    f"T={T}, 2 of 4 KV heads streaming per layer, S={wl.sink} W={wl.window}; one layer timed",
+        "prefill_ms_per_layer": round(pre_ms, 3), "prefill_tflops": round(flops / (pre_ms * 1e-3) / 1e12, 1),
+        "prefill_frac_of_peak": round(flops / (pre_ms * 1e-3) / 1e12 / tf_peak, 4),
+        "decode_us_per_layer_step": round(us, 2), "decode_hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
+        "decode_frac_of_peak": round(nbytes / (us * 1e-6) / 1e9 / hbm, 4),
+        "stack_estimate": {"prefill_s": round(wl.layers * pre_ms / 1000, 3),
+                           "decode_ms_per_token": round(wl.layers * us / 1000, 3)},
+        "kv_bytes_stack": kv_aoh, "kv_bytes_all_retrieval": kv_full, "kv_ratio": round(kv_full / kv_aoh, 4),
+        "peak_note": note}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -451,6 +595,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--prefill-steps", type=int, default=10)
+    ap.add_argument("--prefill-chunks", type=int, default=8)
+    ap.add_argument("--workload", choices=["default", "ragged", "stack"], default="default",
+                    help="default: the headline decode + prefill run; ragged / stack: the other two workloads")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--decode-batch", type=int, default=None, help="smaller decode batch (profiling runs)")
@@ -461,6 +608,10 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "ragged":
+        run_ragged(args)
+    elif args.workload == "stack":
+        run_stack(args)
     else:
         run_native(args)
 

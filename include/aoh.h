@@ -179,7 +179,7 @@ const char* aoh_last_error(void);
  * the handle API for decode. This call runs the same split-KV decode kernel
  * as aoh_decode_step with no handle and performs no device allocation: its
  * scratch (split partials, arrival counters, an error word) lives in one
- * statically allocated device array of 16 MiB + 64 KiB inside the library,
+ * statically allocated device array of 16 MiB + 128 KiB inside the library,
  * which every GPU that loads the library holds until the process exits.
  *
  *   cfg, head_labels  as for aoh_cache_init (host memory, not retained).

@@ -116,6 +116,7 @@ struct aoh_cache {
   int32_t* d_lens = nullptr;
   int32_t* d_chunk = nullptr;  // rows of the current prefill chunk
   uint32_t* d_counters = nullptr;
+  uint32_t* d_gcounters = nullptr;
   uint32_t* d_done = nullptr;
   uint32_t* d_err = nullptr;
   float* d_partials = nullptr;
@@ -191,7 +192,8 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   const size_t n_lens = ((size_t)c.batch + 63) / 64 * 64;
   const size_t n_cnt = ((size_t)c.batch * c.n_kv_heads + 63) / 64 * 64;
   const size_t n_part = decode_partial_floats(2 * h->num_sms, G, c.d_head);
-  const size_t meta_bytes = (2 * n_lens + n_cnt + 64) * 4 + n_part * 4;
+  const size_t n_gcnt = ((size_t)4 * h->num_sms + 63) / 64 * 64;
+  const size_t meta_bytes = (2 * n_lens + n_cnt + n_gcnt + 64) * 4 + n_part * 4;
   e = cudaMalloc(&h->meta, meta_bytes);
   if (e == cudaSuccess) e = cudaMemset(h->meta, 0, meta_bytes);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -204,9 +206,10 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   h->d_lens = reinterpret_cast<int32_t*>(base);
   h->d_chunk = reinterpret_cast<int32_t*>(base + n_lens);
   h->d_counters = base + 2 * n_lens;
-  h->d_done = h->d_counters + n_cnt;
+  h->d_gcounters = h->d_counters + n_cnt;
+  h->d_done = h->d_gcounters + n_gcnt;
   h->d_err = h->d_done + 32;
-  h->d_partials = reinterpret_cast<float*>(base + 2 * n_lens + n_cnt + 64);
+  h->d_partials = reinterpret_cast<float*>(base + 2 * n_lens + n_cnt + n_gcnt + 64);
   *out = h;
   return AOH_OK;
 }
@@ -362,6 +365,7 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
   a.lens = cache->d_lens;
   a.partials = cache->d_partials;
   a.counters = cache->d_counters;
+  a.gcounters = cache->d_gcounters;
   a.done = cache->d_done;
   a.err = cache->d_err;
   a.n_ctas = decode_ctas(total, cache->num_sms);

@@ -101,6 +101,53 @@ __device__ __forceinline__ void reduce_scatter(float (&x)[V], int c) {
   }
 }
 
+constexpr int kGroup = 16;  // parts merged per first-level group
+
+// Merge n partial states (o[G][D] unnormalised, then m[G], l[G]; part(j)
+// returns the j-th) with log-sum-exp weights. Writes the normalised bf16
+// output to `out`, or the merged partial to `dst`. Run by the NW consumer
+// warps; `scratch` holds n*G weights plus 2*G floats of shared memory.
+template <class C, class PartFn>
+__device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch) {
+  constexpr int G = C::G, D = C::D, NT = C::NW * 32;
+  float* wts = scratch;          // [n][G]
+  float* Ls = scratch + n * G;   // [G]
+  float* Ms = Ls + G;            // [G]
+  for (int t = threadIdx.x; t < n * G; t += NT) wts[t] = __ldcg(part(t / G) + G * D + (t % G));
+  named_barrier_sync(1, NT);
+  if (threadIdx.x < G) {
+    const int r = threadIdx.x;
+    float M = -INFINITY;
+    for (int j = 0; j < n; ++j) M = fmaxf(M, wts[j * G + r]);
+    float L = 0.f;
+    for (int j = 0; j < n; ++j) {
+      const float mj = wts[j * G + r];
+      const float w = (mj == -INFINITY) ? 0.f : fast_exp2(mj - M);
+      wts[j * G + r] = w;
+      L += w * __ldcg(part(j) + G * D + G + r);
+    }
+    Ls[r] = L;
+    Ms[r] = M;
+  }
+  named_barrier_sync(1, NT);
+  for (int idx = threadIdx.x; idx < G * D; idx += NT) {
+    const int r = idx / D;
+    float O = 0.f;
+#pragma unroll 4
+    for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
+    if (out) {
+      out[idx] = __float2bfloat16_rn(O / Ls[r]);
+    } else {
+      __stcg(dst + idx, O);
+      if (idx - r * D == 0) {
+        __stcg(dst + G * D + r, Ms[r]);
+        __stcg(dst + G * D + G + r, Ls[r]);
+      }
+    }
+  }
+  named_barrier_sync(1, NT);
+}
+
 // Rows of item `id` (items are ordered b-major: the retrieval heads of a
 // sequence, then its streaming heads). Retrieval: t + 1 rows; streaming:
 // min(t + 1, S + W) ring rows; t = tokens held before this step.
@@ -426,7 +473,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
       const int f = cta_of(item_off, total, P), lst = cta_of(item_off + rows - 1, total, P);
       const bool single = f == lst;
       const int slot = (p == f) ? 1 : 0;
-      float* pbase = a.partials + ((size_t)p * 2 + slot) * (size_t)(G * (D + 2));
+      float* pbase = a.partials + ((size_t)p * 4 + slot) * (size_t)(G * (D + 2));
       bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * D;
       for (int idx = threadIdx.x; idx < G * D; idx += C::NW * 32) {
         const int r = idx / D, d = idx - r * D;
@@ -452,34 +499,52 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
         }
       }
       if (!single) {
+        // Two-level merge of the item's parts (CTAs f..lst). Level 1: groups
+        // of kGroup consecutive CTAs; the last to arrive in a group merges its
+        // group into a group partial (slot 2 or 3 of the group's first CTA).
+        // Level 2: the last group to finish merges the group partials and
+        // writes the output. A one-group item writes the output at level 1.
         __threadfence();
         named_barrier_sync(1, C::NW * 32);
+        const int np = lst - f + 1;
+        const int gi = (p - f) / kGroup, p0 = f + gi * kGroup;
+        const int gsz = min(kGroup, lst - p0 + 1);
+        const int n_groups = (np + kGroup - 1) / kGroup;
+        const int gslot = (p0 == f) ? 1 : 0;  // item i is p0's last item iff p0 == f
         if (threadIdx.x == 0) {
-          const uint32_t prev = atomicAdd(&a.counters[id], 1u);
-          sh32[1] = (prev == (uint32_t)(lst - f));
+          const uint32_t prev = atomicAdd(&a.gcounters[p0 * 2 + gslot], 1u);
+          sh32[1] = (prev == (uint32_t)(gsz - 1));
         }
         named_barrier_sync(1, C::NW * 32);
         if (sh32[1]) {
-          // last part of this item to finish: merge the parts of CTAs f..lst
           __threadfence();
-          for (int idx = threadIdx.x; idx < G * D; idx += C::NW * 32) {
-            const int r = idx / D;
-            float M = -INFINITY;
-            for (int q = f; q <= lst; ++q) {
-              const float* pb = a.partials + ((size_t)q * 2 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
-              M = fmaxf(M, __ldcg(pb + G * D + r));
+          if (threadIdx.x == 0) a.gcounters[p0 * 2 + gslot] = 0u;
+          auto own = [&](int j) {
+            const int q = p0 + j;
+            return a.partials + ((size_t)q * 4 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
+          };
+          if (n_groups == 1) {
+            merge_parts<C>(gsz, own, outp, nullptr, mo);
+          } else {
+            float* gpart = a.partials + ((size_t)p0 * 4 + 2 + gslot) * (size_t)(G * (D + 2));
+            merge_parts<C>(gsz, own, nullptr, gpart, mo);
+            __threadfence();
+            named_barrier_sync(1, C::NW * 32);
+            if (threadIdx.x == 0) {
+              const uint32_t prev = atomicAdd(&a.counters[id], 1u);
+              sh32[1] = (prev == (uint32_t)(n_groups - 1));
             }
-            float O = 0.f, L = 0.f;
-            for (int q = f; q <= lst; ++q) {
-              const float* pb = a.partials + ((size_t)q * 2 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
-              const float mq = __ldcg(pb + G * D + r);
-              const float wt = (mq == -INFINITY) ? 0.f : fast_exp2(mq - M);
-              O += wt * __ldcg(pb + idx);
-              L += wt * __ldcg(pb + G * D + G + r);
+            named_barrier_sync(1, C::NW * 32);
+            if (sh32[1]) {
+              __threadfence();
+              if (threadIdx.x == 0) a.counters[id] = 0u;
+              auto grp_part = [&](int j) {
+                const int q = f + j * kGroup;
+                return a.partials + ((size_t)q * 4 + 2 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
+              };
+              merge_parts<C>(n_groups, grp_part, outp, nullptr, mo);
             }
-            outp[idx] = __float2bfloat16_rn(O / L);
           }
-          if (threadIdx.x == 0) a.counters[id] = 0u;
         }
       }
       named_barrier_sync(1, C::NW * 32);
@@ -528,7 +593,7 @@ int decode_ctas(long long total_rows, int num_sms) {
   return p < 1 ? 1 : (int)p;
 }
 
-size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 2 * G * (D + 2); }
+size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 4 * G * (D + 2); }
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;

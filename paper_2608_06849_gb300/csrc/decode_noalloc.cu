@@ -8,7 +8,7 @@
 // cannot use the handle API for decode. This entry point runs the same
 // split-KV decode kernel, but its scratch (split partials, arrival counters,
 // the error word) lives in one statically allocated device array of this
-// file, sized kNoAllocScratchBytes. Every GPU that loads the library holds
+// file, sized kNoAllocScratchBytes (16 MiB + 128 KiB). Every GPU that loads the library holds
 // that array until the process exits.
 //
 // The array's host-side name is only a stand-in for the device symbol, so the
@@ -25,10 +25,12 @@
 namespace aoh {
 namespace {
 
-constexpr size_t kNoAllocHeaderBytes = 64 * 1024;         // err, done, per-(b, head) counters
+constexpr size_t kNoAllocHeaderBytes = 128 * 1024;        // err, done, item and group counters
 constexpr size_t kNoAllocPartialBytes = 16u * 1024 * 1024;  // split-KV partials
 constexpr size_t kNoAllocScratchBytes = kNoAllocHeaderBytes + kNoAllocPartialBytes;
-constexpr int kNoAllocMaxItems = (int)(kNoAllocHeaderBytes / 4) - 64;  // B * n_kv_heads limit
+constexpr int kNoAllocMaxItems = 16320;  // B * n_kv_heads limit
+constexpr int kNoAllocMaxCtas = 2048;    // decode CTAs (two group counters each)
+static_assert(64 + kNoAllocMaxItems + 2 * kNoAllocMaxCtas <= (int)(kNoAllocHeaderBytes / 4), "header");
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
@@ -121,9 +123,6 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   }
   uint32_t* header = static_cast<uint32_t*>(scratch);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // err, done and the arrival counters must start at zero; clear them every call.
-  e = cudaMemsetAsync(header, 0, (size_t)(64 + items) * 4, s);
-  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaMemsetAsync failed");
 
   // CTA count as the handle API computes it (from an upper bound of the rows),
   // bounded by the partial space.
@@ -133,6 +132,10 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   int n_ctas = decode_ctas(total, num_sms);
   const int cap_ctas = (int)(kNoAllocPartialBytes / (decode_partial_floats(1, G, c.d_head) * 4));
   if (n_ctas > cap_ctas) n_ctas = cap_ctas;
+  if (n_ctas > kNoAllocMaxCtas) n_ctas = kNoAllocMaxCtas;
+  // err, done and the arrival counters must start at zero; clear them every call.
+  e = cudaMemsetAsync(header, 0, (size_t)(64 + items + 2 * n_ctas) * 4, s);
+  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaMemsetAsync failed");
 
   DecodeArgs a;
   a.geom = g;
@@ -145,6 +148,7 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   a.err = header;
   a.done = header + 32;
   a.counters = header + 64;
+  a.gcounters = header + 64 + items;
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
   a.n_ctas = n_ctas;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));

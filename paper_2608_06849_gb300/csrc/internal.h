@@ -43,8 +43,10 @@ struct DecodeArgs {
   void* out;          // [B][Hq][D]
   void* kv;           // cache base
   int32_t* lens;      // [B] tokens held before this step (device)
-  float* partials;    // [n_ctas][2][G][D + 2]: a CTA's first and last shared item
-  uint32_t* counters; // [B][n_r + n_s] arrivals per item (items b-major, retrieval first)
+  float* partials;    // [n_ctas][4][G][D + 2]: a CTA's own partial of its first / last
+                      // shared item, then group partials of those items
+  uint32_t* counters; // [B][n_r + n_s] group arrivals per item (items b-major, retrieval first)
+  uint32_t* gcounters;  // [n_ctas][2] part arrivals per group (indexed by the group's first CTA)
   uint32_t* done;     // CTAs finished in this launch
   uint32_t* err;      // error word
   int n_ctas;         // CTAs sharing the rows of all items equally
