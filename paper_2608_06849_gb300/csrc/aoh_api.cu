@@ -103,6 +103,7 @@ size_t bytes_for(const aoh_config& c, int n_r, int n_s) {
 void aoh::record_error(const char* msg) { g_last_error = msg; }
 
 struct aoh_cache {
+  CUtensorMap tcr, tcs;  // cache regions for TMA (built once: the buffer does not move)
   aoh_config cfg;
   CacheGeom geom;
   std::vector<uint8_t> labels;
@@ -210,6 +211,11 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   h->d_done = h->d_gcounters + n_gcnt;
   h->d_err = h->d_done + 32;
   h->d_partials = reinterpret_cast<float*>(base + 2 * n_lens + n_cnt + n_gcnt + 64);
+  if (!make_cache_region_maps(&h->tcr, &h->tcs, h->geom, h->kv)) {
+    cudaFree(h->meta);
+    delete h;
+    return fail(AOH_ERR_CUDA, "cuTensorMapEncodeTiled failed for the cache regions");
+  }
   *out = h;
   return AOH_OK;
 }
@@ -356,6 +362,8 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
     total += g.n_r * t1 + g.n_s * std::min<long long>(t1, g.S + g.W);
   }
   DecodeArgs a;
+  a.tcr = cache->tcr;
+  a.tcs = cache->tcs;
   a.geom = g;
   a.q = q;
   a.k_new = k_new;
@@ -368,7 +376,7 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
   a.gcounters = cache->d_gcounters;
   a.done = cache->d_done;
   a.err = cache->d_err;
-  a.n_ctas = decode_ctas(total, cache->num_sms);
+  a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
   cudaError_t e = launch_decode(a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");

@@ -26,6 +26,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "decode_common.cuh"
 #include "internal.h"
 
 namespace aoh {
@@ -101,69 +102,6 @@ __device__ __forceinline__ void reduce_scatter(float (&x)[V], int c) {
   }
 }
 
-constexpr int kGroup = 16;  // parts merged per first-level group
-
-// Merge n partial states (o[G][D] unnormalised, then m[G], l[G]; part(j)
-// returns the j-th) with log-sum-exp weights. Writes the normalised bf16
-// output to `out`, or the merged partial to `dst`. Run by the NW consumer
-// warps; `scratch` holds n*G weights plus 2*G floats of shared memory.
-template <class C, class PartFn>
-__device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch) {
-  constexpr int G = C::G, D = C::D, NT = C::NW * 32;
-  float* wts = scratch;          // [n][G]
-  float* Ls = scratch + n * G;   // [G]
-  float* Ms = Ls + G;            // [G]
-  for (int t = threadIdx.x; t < n * G; t += NT) wts[t] = __ldcg(part(t / G) + G * D + (t % G));
-  named_barrier_sync(1, NT);
-  if (threadIdx.x < G) {
-    const int r = threadIdx.x;
-    float M = -INFINITY;
-    for (int j = 0; j < n; ++j) M = fmaxf(M, wts[j * G + r]);
-    float L = 0.f;
-    for (int j = 0; j < n; ++j) {
-      const float mj = wts[j * G + r];
-      const float w = (mj == -INFINITY) ? 0.f : fast_exp2(mj - M);
-      wts[j * G + r] = w;
-      L += w * __ldcg(part(j) + G * D + G + r);
-    }
-    Ls[r] = L;
-    Ms[r] = M;
-  }
-  named_barrier_sync(1, NT);
-  for (int idx = threadIdx.x; idx < G * D; idx += NT) {
-    const int r = idx / D;
-    float O = 0.f;
-#pragma unroll 4
-    for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
-    if (out) {
-      out[idx] = __float2bfloat16_rn(O / Ls[r]);
-    } else {
-      __stcg(dst + idx, O);
-      if (idx - r * D == 0) {
-        __stcg(dst + G * D + r, Ms[r]);
-        __stcg(dst + G * D + G + r, Ls[r]);
-      }
-    }
-  }
-  named_barrier_sync(1, NT);
-}
-
-// Rows of item `id` (items are ordered b-major: the retrieval heads of a
-// sequence, then its streaming heads). Retrieval: t + 1 rows; streaming:
-// min(t + 1, S + W) ring rows; t = tokens held before this step.
-__device__ __forceinline__ int item_rows(const DecodeArgs& a, int id) {
-  const CacheGeom& g = a.geom;
-  const int HK = g.n_r + g.n_s;
-  const int b = id / HK, k = id - b * HK;
-  const int t = __ldcg(&a.lens[b]);
-  return k < g.n_r ? t + 1 : min(t + 1, g.S + g.W);
-}
-
-// CTA whose row range contains global row x (ranges [p*T/P, (p+1)*T/P)).
-__device__ __forceinline__ int cta_of(long long x, long long total, int P) {
-  return (int)(((x + 1) * (long long)P - 1) / total);
-}
-
 template <class C>
 __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constant__ DecodeArgs a) {
   constexpr int D = C::D, G = C::G, RB = C::RB, TOK = C::TOK, NST = C::NST;
@@ -183,54 +121,19 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
   const int n_items = g.B * HK;
   const int P = a.n_ctas, p = blockIdx.x;
 
-  // ---- prefix sums of the items' rows: every CTA finds its share of the
-  // concatenated rows [p * total / P, (p + 1) * total / P) and the first item
-  // it touches. The ring memory is scratch here.
-  {
-    long long* part = reinterpret_cast<long long*>(smem);
-    const int per = (n_items + C::THREADS - 1) / C::THREADS;
-    const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
-    long long mine = 0;
-    for (int id = i0; id < i1; ++id) mine += item_rows(a, id);
-    part[threadIdx.x] = mine;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      long long run = 0;
-      for (int t = 0; t < C::THREADS; ++t) {
-        const long long v = part[t];
-        part[t] = run;
-        run += v;
-      }
-      sh64[0] = run;
-      sh32[0] = n_items;
-      sh64[1] = run;
-    }
-    __syncthreads();
-    const long long total = sh64[0];
-    const long long start = (long long)p * total / P;
-    long long off = part[threadIdx.x];
-    if (i0 < i1 && off <= start && start < off + mine) {
-      int id = i0;
-      while (true) {
-        const int r = item_rows(a, id);
-        if (start < off + r) break;
-        off += r;
-        ++id;
-      }
-      sh32[0] = id;
-      sh64[1] = off;
-    }
-    if (threadIdx.x == 0) {
+  // ---- every CTA finds its share of the concatenated rows and the first
+  // item it touches (the ring memory is scratch here)
+  dec::find_cta_range<C::THREADS>(a, reinterpret_cast<long long*>(smem), sh64, sh32);
+  if (threadIdx.x == 0) {
 #pragma unroll
-      for (int s = 0; s < NST; ++s) {
-        mbar_init(&full[s], 1);
-        mbar_init(&empty[s], C::NW);
-      }
-      *abort_flag = 0;
-      fence_mbar_init();
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], C::NW);
     }
-    __syncthreads();
+    *abort_flag = 0;
+    fence_mbar_init();
   }
+  __syncthreads();
   const long long total = sh64[0];
   const long long start = (long long)p * total / P;
   const long long end = (long long)(p + 1) * total / P;
@@ -242,7 +145,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
     int it = 0;
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end; ++id) {
-      const int rows = item_rows(a, id);
+      const int rows = dec::item_rows(a, id);
       const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
       off += rows;
       if (lo >= hi) continue;
@@ -292,7 +195,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
     int it = 0;
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end; ++id) {
-      const int rows = item_rows(a, id);
+      const int rows = dec::item_rows(a, id);
       const long long item_off = off;
       const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
       off += rows;
@@ -470,10 +373,10 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
       }
       named_barrier_sync(1, C::NW * 32);
 
-      const int f = cta_of(item_off, total, P), lst = cta_of(item_off + rows - 1, total, P);
+      const int f = dec::cta_of(item_off, total, P), lst = dec::cta_of(item_off + rows - 1, total, P);
       const bool single = f == lst;
       const int slot = (p == f) ? 1 : 0;
-      float* pbase = a.partials + ((size_t)p * 4 + slot) * (size_t)(G * (D + 2));
+      float* pbase = dec::partial_slot(a, p, slot, G, D);
       bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * D;
       for (int idx = threadIdx.x; idx < G * D; idx += C::NW * 32) {
         const int r = idx / D, d = idx - r * D;
@@ -498,70 +401,14 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
           }
         }
       }
-      if (!single) {
-        // Two-level merge of the item's parts (CTAs f..lst). Level 1: groups
-        // of kGroup consecutive CTAs; the last to arrive in a group merges its
-        // group into a group partial (slot 2 or 3 of the group's first CTA).
-        // Level 2: the last group to finish merges the group partials and
-        // writes the output. A one-group item writes the output at level 1.
-        __threadfence();
-        named_barrier_sync(1, C::NW * 32);
-        const int np = lst - f + 1;
-        const int gi = (p - f) / kGroup, p0 = f + gi * kGroup;
-        const int gsz = min(kGroup, lst - p0 + 1);
-        const int n_groups = (np + kGroup - 1) / kGroup;
-        const int gslot = (p0 == f) ? 1 : 0;  // item i is p0's last item iff p0 == f
-        if (threadIdx.x == 0) {
-          const uint32_t prev = atomicAdd(&a.gcounters[p0 * 2 + gslot], 1u);
-          sh32[1] = (prev == (uint32_t)(gsz - 1));
-        }
-        named_barrier_sync(1, C::NW * 32);
-        if (sh32[1]) {
-          __threadfence();
-          if (threadIdx.x == 0) a.gcounters[p0 * 2 + gslot] = 0u;
-          auto own = [&](int j) {
-            const int q = p0 + j;
-            return a.partials + ((size_t)q * 4 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
-          };
-          if (n_groups == 1) {
-            merge_parts<C>(gsz, own, outp, nullptr, mo);
-          } else {
-            float* gpart = a.partials + ((size_t)p0 * 4 + 2 + gslot) * (size_t)(G * (D + 2));
-            merge_parts<C>(gsz, own, nullptr, gpart, mo);
-            __threadfence();
-            named_barrier_sync(1, C::NW * 32);
-            if (threadIdx.x == 0) {
-              const uint32_t prev = atomicAdd(&a.counters[id], 1u);
-              sh32[1] = (prev == (uint32_t)(n_groups - 1));
-            }
-            named_barrier_sync(1, C::NW * 32);
-            if (sh32[1]) {
-              __threadfence();
-              if (threadIdx.x == 0) a.counters[id] = 0u;
-              auto grp_part = [&](int j) {
-                const int q = f + j * kGroup;
-                return a.partials + ((size_t)q * 4 + 2 + (q == f ? 1 : 0)) * (size_t)(G * (D + 2));
-              };
-              merge_parts<C>(n_groups, grp_part, outp, nullptr, mo);
-            }
-          }
-        }
-      }
+      if (!single) dec::merge_item<G, D, C::NW * 32>(a, p, f, lst, id, outp, mo, sh32 + 1);
       named_barrier_sync(1, C::NW * 32);
     }
   }
 
   // ---- the launch's last CTA advances the lengths
   __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    const uint32_t prev = atomicAdd(a.done, 1u);
-    if (prev == gridDim.x - 1) {
-      for (int i = 0; i < g.B; ++i) a.lens[i] += 1;
-      __threadfence();
-      *a.done = 0u;
-    }
-  }
+  if (threadIdx.x == 0) dec::finish_launch(a);
 }
 
 template <int D, int G>
@@ -586,7 +433,8 @@ bool decode_supported(int D, int G) {
 
 // Two CTAs fit on an SM (about 100 KB of shared memory each), so 2 x SMs
 // CTAs run as one wave; small launches use fewer, at least 256 rows each.
-int decode_ctas(long long total_rows, int num_sms) {
+int decode_ctas(long long total_rows, int num_sms, int D, int G) {
+  if (decode_uses_tc(D, G)) return decode_tc_ctas(total_rows, num_sms);
   const long long by_rows = (total_rows + 255) / 256;
   long long p = 2LL * num_sms;
   if (by_rows < p) p = by_rows;
@@ -597,6 +445,7 @@ size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas *
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;
+  if (decode_uses_tc(D, G)) return launch_decode_tc(a, s);
   if (D == 128) {
     switch (G) {
       case 1: return launch_cfg<128, 1>(a, s);

@@ -1,0 +1,196 @@
+// Pieces shared by the two decode kernels (CUDA cores, tcgen05): the
+// stream-K split of a step's cached rows over the CTAs of a launch, and the
+// merge of an item's split partials (Sec. 5 "Decode Stage": each head's
+// softmax over its visible positions, assembled from per-split
+// log-sum-exp states).
+//
+// An item is one (sequence b, KV head) pair; items are ordered b-major, the
+// retrieval heads of a sequence before its streaming heads. The rows of all
+// items are concatenated and CTA p of P takes rows [p*T/P, (p+1)*T/P).
+#pragma once
+
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace aoh {
+namespace dec {
+
+constexpr int kGroup = 16;  // parts merged per first-level group
+
+// Rows of item `id`. Retrieval: t + 1 rows; streaming: min(t + 1, S + W)
+// ring rows; t = tokens held before this step.
+__device__ __forceinline__ int item_rows(const DecodeArgs& a, int id) {
+  const CacheGeom& g = a.geom;
+  const int HK = g.n_r + g.n_s;
+  const int b = id / HK, k = id - b * HK;
+  const int t = __ldcg(&a.lens[b]);
+  return k < g.n_r ? t + 1 : min(t + 1, g.S + g.W);
+}
+
+// CTA whose row range contains global row x.
+__device__ __forceinline__ int cta_of(long long x, long long total, int P) {
+  return (int)(((x + 1) * (long long)P - 1) / total);
+}
+
+// Block-wide prefix sum of the items' rows. On return (after the caller's
+// next __syncthreads) sh64[0] = total rows, sh64[1] = first row of the first
+// item this CTA touches, sh32[0] = that item. `part` is THREADS longs of
+// scratch shared memory.
+template <int THREADS>
+__device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* part, long long* sh64, int* sh32) {
+  const CacheGeom& g = a.geom;
+  const int n_items = g.B * (g.n_r + g.n_s);
+  const int P = a.n_ctas, p = blockIdx.x;
+  const int per = (n_items + THREADS - 1) / THREADS;
+  const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
+  long long mine = 0;
+  for (int id = i0; id < i1; ++id) mine += item_rows(a, id);
+  part[threadIdx.x] = mine;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long run = 0;
+    for (int t = 0; t < THREADS; ++t) {
+      const long long v = part[t];
+      part[t] = run;
+      run += v;
+    }
+    sh64[0] = run;
+    sh32[0] = n_items;
+    sh64[1] = run;
+  }
+  __syncthreads();
+  const long long total = sh64[0];
+  const long long start = (long long)p * total / P;
+  long long off = part[threadIdx.x];
+  if (i0 < i1 && off <= start && start < off + mine) {
+    int id = i0;
+    while (true) {
+      const int r = item_rows(a, id);
+      if (start < off + r) break;
+      off += r;
+      ++id;
+    }
+    sh32[0] = id;
+    sh64[1] = off;
+  }
+}
+
+// Partial state of split CTA q for an item whose first CTA is f: o[G][D]
+// (unnormalised), then m[G] (running max, log2 units), then l[G]. Slot 0/1:
+// the CTA's first / last shared item; slot 2/3: the group partial of the
+// group the CTA heads.
+__device__ __forceinline__ float* partial_slot(const DecodeArgs& a, int q, int slot, int G, int D) {
+  return a.partials + ((size_t)q * 4 + slot) * (size_t)(G * (D + 2));
+}
+
+// Merge n partial states (part(j) returns the j-th) with log-sum-exp
+// weights. Writes the normalised bf16 output to `out`, or the merged partial
+// to `dst`. Run by NT threads that share named barrier 1; `scratch` holds
+// n*G + 2*G floats of shared memory.
+template <int G, int D, int NT, class PartFn>
+__device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch) {
+  float* wts = scratch;          // [n][G]
+  float* Ls = scratch + n * G;   // [G]
+  float* Ms = Ls + G;            // [G]
+  for (int t = threadIdx.x; t < n * G; t += NT) wts[t] = __ldcg(part(t / G) + G * D + (t % G));
+  named_barrier_sync(1, NT);
+  if (threadIdx.x < G) {
+    const int r = threadIdx.x;
+    float M = -INFINITY;
+    for (int j = 0; j < n; ++j) M = fmaxf(M, wts[j * G + r]);
+    float L = 0.f;
+    for (int j = 0; j < n; ++j) {
+      const float mj = wts[j * G + r];
+      const float w = (mj == -INFINITY) ? 0.f : fast_exp2(mj - M);
+      wts[j * G + r] = w;
+      L += w * __ldcg(part(j) + G * D + G + r);
+    }
+    Ls[r] = L;
+    Ms[r] = M;
+  }
+  named_barrier_sync(1, NT);
+  for (int idx = threadIdx.x; idx < G * D; idx += NT) {
+    const int r = idx / D;
+    float O = 0.f;
+#pragma unroll 4
+    for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
+    if (out) {
+      out[idx] = __float2bfloat16_rn(O / Ls[r]);
+    } else {
+      __stcg(dst + idx, O);
+      if (idx - r * D == 0) {
+        __stcg(dst + G * D + r, Ms[r]);
+        __stcg(dst + G * D + G + r, Ls[r]);
+      }
+    }
+  }
+  named_barrier_sync(1, NT);
+}
+
+// After CTA p wrote its partial of item `id` (CTAs f..lst share it, f < lst),
+// merge in two levels. Level 1: groups of kGroup consecutive CTAs; the last
+// to arrive in a group merges the group into a group partial (slot 2 or 3 of
+// the group's first CTA). Level 2: the last group to finish merges the group
+// partials and writes the output. A one-group item writes the output at
+// level 1. Run by the NT threads that wrote the partial; `flag` is one int
+// of shared memory, `scratch` as for merge_parts.
+template <int G, int D, int NT>
+__device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, int lst, int id,
+                                           __nv_bfloat16* outp, float* scratch, volatile int* flag) {
+  __threadfence();
+  named_barrier_sync(1, NT);
+  const int np = lst - f + 1;
+  const int gi = (p - f) / kGroup, p0 = f + gi * kGroup;
+  const int gsz = min(kGroup, lst - p0 + 1);
+  const int n_groups = (np + kGroup - 1) / kGroup;
+  const int gslot = (p0 == f) ? 1 : 0;  // the item is p0's last item iff p0 == f
+  if (threadIdx.x == 0) {
+    const uint32_t prev = atomicAdd(&a.gcounters[p0 * 2 + gslot], 1u);
+    *flag = (prev == (uint32_t)(gsz - 1));
+  }
+  named_barrier_sync(1, NT);
+  if (!*flag) return;
+  __threadfence();
+  if (threadIdx.x == 0) a.gcounters[p0 * 2 + gslot] = 0u;
+  auto own = [&](int j) {
+    const int q = p0 + j;
+    return partial_slot(a, q, q == f ? 1 : 0, G, D);
+  };
+  if (n_groups == 1) {
+    merge_parts<G, D, NT>(gsz, own, outp, nullptr, scratch);
+    return;
+  }
+  merge_parts<G, D, NT>(gsz, own, nullptr, partial_slot(a, p0, 2 + gslot, G, D), scratch);
+  __threadfence();
+  named_barrier_sync(1, NT);
+  if (threadIdx.x == 0) {
+    const uint32_t prev = atomicAdd(&a.counters[id], 1u);
+    *flag = (prev == (uint32_t)(n_groups - 1));
+  }
+  named_barrier_sync(1, NT);
+  if (!*flag) return;
+  __threadfence();
+  if (threadIdx.x == 0) a.counters[id] = 0u;
+  auto grp_part = [&](int j) {
+    const int q = f + j * kGroup;
+    return partial_slot(a, q, 2 + (q == f ? 1 : 0), G, D);
+  };
+  merge_parts<G, D, NT>(n_groups, grp_part, outp, nullptr, scratch);
+}
+
+// The launch's last CTA advances every sequence length by one. Called by
+// thread 0 after a __syncthreads that follows all of the CTA's work.
+__device__ __forceinline__ void finish_launch(const DecodeArgs& a) {
+  __threadfence();
+  const uint32_t prev = atomicAdd(a.done, 1u);
+  if (prev == gridDim.x - 1) {
+    for (int i = 0; i < a.geom.B; ++i) a.lens[i] += 1;
+    __threadfence();
+    *a.done = 0u;
+  }
+}
+
+}  // namespace dec
+}  // namespace aoh

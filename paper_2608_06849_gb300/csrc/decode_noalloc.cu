@@ -129,7 +129,7 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   const long long t1 = (long long)max_len + 1;
   const long long win = t1 < c.sink + c.window ? t1 : c.sink + c.window;
   const long long total = (long long)c.batch * ((long long)n_r * t1 + (long long)n_s * win);
-  int n_ctas = decode_ctas(total, num_sms);
+  int n_ctas = decode_ctas(total, num_sms, c.d_head, G);
   const int cap_ctas = (int)(kNoAllocPartialBytes / (decode_partial_floats(1, G, c.d_head) * 4));
   if (n_ctas > cap_ctas) n_ctas = cap_ctas;
   if (n_ctas > kNoAllocMaxCtas) n_ctas = kNoAllocMaxCtas;
@@ -138,6 +138,8 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaMemsetAsync failed");
 
   DecodeArgs a;
+  if (!make_cache_region_maps(&a.tcr, &a.tcs, g, kv_buffer))
+    return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cuTensorMapEncodeTiled failed");
   a.geom = g;
   a.q = q;
   a.k_new = k_new;

@@ -1,0 +1,488 @@
+// Split-KV decode on tcgen05 tensor cores for large GQA groups (Sec. 5,
+// "Decode Stage", Eq. 8; d_head = 128). With G query heads per KV head, every
+// cached K/V row meets G queries: 4*G*d flops per 4*d bytes. Above g = 4 that
+// arithmetic no longer hides under the HBM stream on CUDA cores, so here it
+// runs as two skinny MMAs per 128-key tile, with the G heads padded to N = 16:
+//
+//   S^T[128 keys][16]  = K_tile[128][d] . Q^T           (A = K, K-major; B = Q, K-major)
+//   O^T[d][16]        += V_tile^T[d][128] . P^T[128][16] (A = V, MN-major; B = P, K-major)
+//
+// Both accumulators live in TMEM: S^T in one of two 16-column buffers (row =
+// key), O^T in 16 more columns (row = d). The split of the step's rows over
+// CTAs, the partial format and the merge are those of the CUDA-core kernel
+// (decode_common.cuh); one CTA per SM.
+//
+// Warp roles (192 threads):
+//   warps 0-3  softmax: thread t owns key t of the tile (TMEM lane t). It
+//              reads its 16 scores, hides keys past the tile's valid rows,
+//              takes the per-head tile maximum (warp redux, then the four
+//              warps through shared memory), moves the running maximum only
+//              when it grows by more than 2^8 (then rescales its row d = t of
+//              O^T in TMEM), forms p = 2^(s - m) and writes P^T as bf16 into a
+//              swizzled K-major [16][128] buffer. Per-thread partial sums of p
+//              are reduced once per item. Rows past the valid keys of a tail V
+//              tile are zeroed first: they may hold unwritten cache rows and a
+//              zero weight times a NaN is NaN.
+//   warp 4     TMA producer: K and V tiles of one (sequence, KV head) region
+//              into a 3-stage ring (4D tensor maps over the cache regions,
+//              128-byte swizzle, rows past the region read as zeros).
+//   warp 5     TMEM owner and MMA issuer. Loads each item's Q into one of two
+//              swizzled buffers, writes the new token's K/V row over its
+//              (stale) cache row in the landed tile and appends it to the
+//              cache, issues S(j) and then O += P(j-1) V(j-1).
+#include <math.h>
+
+#include "common.cuh"
+#include "decode_common.cuh"
+#include "internal.h"
+#include "tc.cuh"
+
+namespace aoh {
+namespace {
+
+using bf16 = __nv_bfloat16;
+constexpr int kD = 128;
+constexpr int kBN = 128;                   // keys per tile
+constexpr int kN = 16;                     // N of both MMAs (query heads, padded)
+constexpr int kNS = 3;                     // ring stages
+constexpr int kThreads = 192;
+constexpr int kSoftmaxThreads = 128;
+constexpr uint32_t kTmemCols = 64;         // S[0] [0,16), S[1] [16,32), O [32,48)
+constexpr uint32_t kOcol = 32;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr int kBox = kBN * 64 * 2;         // one [128 rows][64] TMA box, 16 KB
+constexpr int kTile = 2 * kBox;            // a K or V tile (d = 128)
+constexpr int kStage = 2 * kTile;          // K then V
+constexpr int kOpBuf = 2 * kN * 128;       // [16 rows][128] bf16 operand, two 64-wide blocks
+constexpr int OFF_KV = 0;
+constexpr int OFF_Q = OFF_KV + kNS * kStage;
+constexpr int OFF_P = OFF_Q + 2 * kOpBuf;
+constexpr int OFF_RED = OFF_P + 2 * kOpBuf;   // [2][4][16] warp maxima, [4][16] warp sums
+constexpr int OFF_MS = OFF_RED + (2 * 64 + 64) * 4;
+constexpr int MS_FLOATS = 512;                // merge scratch
+constexpr int OFF_BAR = OFF_MS + MS_FLOATS * 4;
+constexpr int NBAR = 2 * kNS + 2 + 2 + 2 + 2 + 1 + 1;
+constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+constexpr int SMEM = OFF_MISC + 64 + 1024;
+constexpr uint32_t IDESC_S = idesc_bf16(kBN, kN, false, false);
+constexpr uint32_t IDESC_PV = idesc_bf16(kD, kN, false, true);
+static_assert(SMEM <= 232448, "shared memory");
+static_assert(OFF_Q % 1024 == 0 && OFF_P % 1024 == 0, "operand alignment");
+static_assert(kThreads * 8 <= kNS * kStage, "scan scratch");
+
+template <int G>
+__global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
+  static_assert(G >= 1 && G <= kN, "group size");
+  static_assert((dec::kGroup + 8) * G + 2 * G <= MS_FLOATS, "merge scratch");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+  uint8_t* sKV = smem + OFF_KV;
+  uint8_t* sQ = smem + OFF_Q;
+  uint8_t* sP = smem + OFF_P;
+  float* red = reinterpret_cast<float*>(smem + OFF_RED);  // [2][4][16]
+  float* lsum = red + 2 * 64;                             // [4][16]
+  float* ms = reinterpret_cast<float*>(smem + OFF_MS);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  uint64_t* empty = full + kNS;
+  uint64_t* s_full = empty + kNS;   // [2] S(j) in TMEM
+  uint64_t* s_free = s_full + 2;    // [2] S(j) read by the softmax
+  uint64_t* p_full = s_free + 2;    // [2] P(j) written
+  uint64_t* p_free = p_full + 2;    // [2] O += P(j) V(j) done
+  uint64_t* o_free = p_free + 2;    // the item's final O read
+  uint64_t* drain = o_free + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  long long* sh64 = reinterpret_cast<long long*>(smem + OFF_MISC + 8);  // [0] total, [1] first offset
+  int* sh32 = reinterpret_cast<int*>(sh64 + 2);                         // [0] first item, [1] merge flag
+
+  const CacheGeom& g = a.geom;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int HK = g.n_r + g.n_s;
+  const int n_items = g.B * HK;
+  const int P = a.n_ctas, p = blockIdx.x;
+
+  dec::find_cta_range<kThreads>(a, reinterpret_cast<long long*>(sKV), sh64, sh32);
+  // Q and P rows >= G stay zero for the whole launch
+  for (int i = threadIdx.x; i < 4 * kOpBuf / 16; i += kThreads)
+    reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0, 0, 0, 0);
+  fence_proxy_async_smem();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kNS; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&s_full[x], 1);
+      mbar_init(&s_free[x], 4);
+      mbar_init(&p_full[x], 4);
+      mbar_init(&p_free[x], 1);
+    }
+    mbar_init(o_free, 4);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 5) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const long long total = sh64[0];
+  const long long start = (long long)p * total / P;
+  const long long end = (long long)(p + 1) * total / P;
+  const int first_id = sh32[0];
+  const long long first_off = sh64[1];
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      if (g.n_r > 0) prefetch_tmap(&a.tcr);
+      if (g.n_s > 0) prefetch_tmap(&a.tcs);
+      int it = 0;
+      bool ok = true;
+      long long off = first_off;
+      for (int id = first_id; id < n_items && off < end && ok; ++id) {
+        const int rows = dec::item_rows(a, id);
+        const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
+        off += rows;
+        if (lo >= hi) continue;
+        const int b = id / HK, k = id - b * HK;
+        const bool strm = k >= g.n_r;
+        const int region = strm ? b * g.n_s + (k - g.n_r) : b * g.n_r + k;
+        const CUtensorMap* map = strm ? &a.tcs : &a.tcr;
+        for (int row0 = lo; row0 < hi; row0 += kBN) {
+          const int st = it % kNS;
+          if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[st], kStage);
+          uint8_t* dst = sKV + st * kStage;
+#pragma unroll
+          for (int sel = 0; sel < 2; ++sel)
+#pragma unroll
+            for (int db = 0; db < 2; ++db)
+              tma_load_4d(dst + sel * kTile + db * kBox, map, db * 64, row0, sel, region, &full[st]);
+          ++it;
+        }
+      }
+      // every issued copy lands before the CTA can exit
+      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) wait_bar(&full[j % kNS], (j / kNS) & 1, a.err, abort_flag);
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------ MMA issuer
+    const uint32_t kv_addr = smem_u32(sKV), q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
+    int it = 0, item_k = 0, ofw = 0;
+    bool ok = true;
+    struct Pend {
+      int it, st, item;
+      bool first;
+    } pend{0, 0, 0, false};
+    bool has_pend = false;
+    auto wait_warp = [&](uint64_t* bar, uint32_t parity) {
+      if (ok) ok = __all_sync(0xffffffffu, wait_bar(bar, parity, a.err, abort_flag));
+    };
+    // o_free phases complete once per item, in order
+    auto wait_ofree = [&](int n) {
+      while (ok && ofw < n) {
+        wait_warp(o_free, ofw & 1);
+        ++ofw;
+      }
+    };
+    auto issue_pv = [&](const Pend& t) {
+      wait_warp(&p_full[t.it & 1], (t.it >> 1) & 1);
+      if (t.first && t.item >= 1) wait_ofree(t.item);  // accumulate = 0 overwrites the last item's O
+      if (!ok) return;
+      if (lane == 0) {
+        tc_fence_after();
+        const uint32_t v_addr = kv_addr + t.st * kStage + kTile;
+        const uint32_t pb = p_addr + (t.it & 1) * kOpBuf;
+#pragma unroll
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(v_addr + kk * 2048, kBox, 1024);
+          const uint64_t bd = sdesc_sw128(pb + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
+          tc_mma(tmem + kOcol, ad, bd, IDESC_PV, (t.first && kk == 0) ? 0u : 1u);
+        }
+        tc_commit(&p_free[t.it & 1]);
+        tc_commit(&empty[t.st]);
+      }
+      __syncwarp();
+    };
+
+    long long off = first_off;
+    for (int id = first_id; id < n_items && off < end && ok; ++id) {
+      const int rows = dec::item_rows(a, id);
+      const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
+      off += rows;
+      if (lo >= hi) continue;
+      const int b = id / HK, k = id - b * HK;
+      const bool strm = k >= g.n_r;
+      const int hi_idx = strm ? k - g.n_r : k;
+      const int kvh = strm ? g.s_head[hi_idx] : g.r_head[hi_idx];
+      const int t = __ldcg(&a.lens[b]);
+      const int cap = strm ? g.S + g.W : g.max_seq;
+      const int xr = strm ? (t < g.S ? t : g.S + (t - g.S) % g.W) : t;  // the new token's row
+      bf16* Kc = static_cast<bf16*>(a.kv) + (strm ? g.s_region(b, hi_idx) : g.r_region(b, hi_idx));
+      bf16* Vc = Kc + (size_t)cap * kD;
+
+      // this item's Q into buffer item_k & 1, last read by the MMAs of item item_k - 2
+      wait_ofree(item_k - 1);
+      if (!ok) break;
+      {
+        const bf16* qg = static_cast<const bf16*>(a.q) + ((size_t)b * g.Hq + (size_t)kvh * G) * kD;
+        uint8_t* qs = sQ + (item_k & 1) * kOpBuf;
+        for (int c = lane; c < G * 16; c += 32) {  // 16-byte chunks: head c / 16, chunk c % 16
+          const int h = c >> 4, cc = c & 15;
+          const uint4 v = *reinterpret_cast<const uint4*>(qg + (size_t)h * kD + cc * 8);
+          *reinterpret_cast<uint4*>(qs + (cc >> 3) * (kN * 128) + h * 128 + (((cc & 7) ^ (h & 7)) << 4)) = v;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+      }
+      // lanes 0-15 hold the new K row's 16-byte chunks, lanes 16-31 the V row's
+      const int ch = lane & 15;
+      const size_t new_off = ((size_t)b * g.Hkv + kvh) * kD + ch * 8;
+      const uint4 nv = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(lane < 16 ? a.k_new : a.v_new) +
+                                                       new_off);
+
+      for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
+        const int st = it % kNS;
+        const int cnt = min(kBN, hi - row0);
+        wait_warp(&full[st], (it / kNS) & 1);
+        if (!ok) break;
+        if (xr >= row0 && xr < row0 + cnt) {
+          const int r = xr - row0;
+          uint8_t* dst = sKV + st * kStage + (lane < 16 ? 0 : kTile) + (ch >> 3) * kBox + r * 128 +
+                         (((ch & 7) ^ (r & 7)) << 4);
+          *reinterpret_cast<uint4*>(dst) = nv;
+          *reinterpret_cast<uint4*>((lane < 16 ? Kc : Vc) + (size_t)xr * kD + ch * 8) = nv;  // append
+          fence_proxy_async_smem();
+          __syncwarp();
+        }
+        if (it >= 2) wait_warp(&s_free[it & 1], ((it >> 1) - 1) & 1);
+        if (!ok) break;
+        if (lane == 0) {
+          tc_fence_after();
+          const uint32_t k_addr = kv_addr + st * kStage;
+          const uint32_t qb = q_addr + (item_k & 1) * kOpBuf;
+#pragma unroll
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint64_t ad = sdesc_sw128(k_addr + (kk >> 2) * kBox + (kk & 3) * 32, 16, 1024);
+            const uint64_t bd = sdesc_sw128(qb + (kk >> 2) * (kN * 128) + (kk & 3) * 32, 16, 1024);
+            tc_mma(tmem + (it & 1) * kN, ad, bd, IDESC_S, kk > 0 ? 1u : 0u);
+          }
+          tc_commit(&s_full[it & 1]);
+        }
+        __syncwarp();
+        if (has_pend) issue_pv(pend);
+        pend = Pend{it, st, item_k, row0 == lo};
+        has_pend = true;
+      }
+      ++item_k;
+    }
+    if (has_pend) issue_pv(pend);
+    if (lane == 0) {
+      tc_commit(drain);
+      wait_bar(drain, 0, a.err, abort_flag);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int t = threadIdx.x;  // key of the tile / row d of O^T
+    const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+    int it = 0;
+    // ok: the four warps' common verdict, only ever set at a barrier (so every
+    // thread leaves the loops together); local_ok: this thread's waits since
+    bool ok = true, local_ok = true;
+    long long off = first_off;
+    for (int id = first_id; id < n_items && off < end && ok; ++id) {
+      const int rows = dec::item_rows(a, id);
+      const long long item_off = off;
+      const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
+      off += rows;
+      if (lo >= hi) continue;
+      const int b = id / HK, k = id - b * HK;
+      const bool strm = k >= g.n_r;
+      const int kvh = strm ? g.s_head[k - g.n_r] : g.r_head[k];
+
+      float m[G], l[G];
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        m[h] = -INFINITY;
+        l[h] = 0.f;
+      }
+      for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
+        const int x = it & 1, st = it % kNS;
+        const int cnt = min(kBN, hi - row0);
+        local_ok = wait_bar(&s_full[x], (it >> 1) & 1, a.err, abort_flag) && local_ok;
+        tc_fence_after();
+        uint32_t v[16];
+        tmem_ld16(tl + x * kN, v);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_free[x]);
+        const bool valid = t < cnt;
+        float s[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) s[h] = valid ? __uint_as_float(v[h]) * a.scale_log2 : -INFINITY;
+
+        // per-head maximum over the tile: each warp, then the four warps
+        float* rx = red + x * 64;
+        float wm = -INFINITY;
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float r = warp_max(s[h]);
+          wm = (lane == h) ? r : wm;
+        }
+        if (lane < G) rx[warp * 16 + lane] = wm;
+        ok = named_barrier_and(1, kSoftmaxThreads, local_ok);
+        if (!ok) break;
+        bool resc = false;
+        float alpha[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float tm = fmaxf(fmax3f(rx[h], rx[16 + h], rx[32 + h]), rx[48 + h]);
+          const float mn = fmaxf(m[h], tm);
+          alpha[h] = 1.f;
+          if (mn > m[h] + kRescaleThreshold) {
+            alpha[h] = (m[h] == -INFINITY) ? 0.f : fast_exp2(m[h] - mn);
+            m[h] = mn;
+            l[h] *= alpha[h];
+            resc = true;
+          }
+        }
+        // P buffer x is free once O += P(it - 2) V is done
+        if (it >= 2) local_ok = wait_bar(&p_free[x], ((it >> 1) - 1) & 1, a.err, abort_flag) && local_ok;
+        if (resc && row0 != lo) {
+          // rescale row t of O^T; O += P(it - 1) V must have landed first
+          local_ok = wait_bar(&p_free[x ^ 1], ((it - 1) >> 1) & 1, a.err, abort_flag) && local_ok;
+          tc_fence_after();
+          uint32_t o[16];
+          tmem_ld16(tl + kOcol, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int h = 0; h < G; ++h) o[h] = __float_as_uint(__uint_as_float(o[h]) * alpha[h]);
+          tmem_st16(tl + kOcol, o);
+          tmem_st_wait();
+        }
+        float pr[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          pr[h] = valid ? fast_exp2(s[h] - m[h]) : 0.f;
+          l[h] += pr[h];
+        }
+        if (!valid) {
+          // the tile has landed (its S is complete); zero V row t
+          wait_bar(&full[st], (it / kNS) & 1, a.err, abort_flag);
+          uint8_t* vr = sKV + st * kStage + kTile + t * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            reinterpret_cast<uint4*>(vr)[c] = make_uint4(0, 0, 0, 0);
+            reinterpret_cast<uint4*>(vr + kBox)[c] = make_uint4(0, 0, 0, 0);
+          }
+        }
+        // P^T row t -> column t of the K-major [16 heads][128 keys] buffer
+        uint8_t* pb = sP + x * kOpBuf + (t >> 6) * (kN * 128) + (t & 7) * 2;
+        const int j = (t & 63) >> 3;
+#pragma unroll
+        for (int h = 0; h < G; ++h)
+          *reinterpret_cast<bf16*>(pb + h * 128 + ((j ^ (h & 7)) << 4)) = __float2bfloat16_rn(pr[h]);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[x]);
+      }
+      if (!ok) break;
+
+      // ---- the item's state: O^T row t, m (uniform), l summed over the keys
+      const int last = it - 1;
+      local_ok = wait_bar(&p_free[last & 1], (last >> 1) & 1, a.err, abort_flag) && local_ok;
+      tc_fence_after();
+      uint32_t o[16];
+      tmem_ld16(tl + kOcol, o);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free);
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        float v = l[h];
+#pragma unroll
+        for (int msk = 16; msk >= 1; msk >>= 1) v += __shfl_xor_sync(0xffffffffu, v, msk);
+        if (lane == 0) lsum[warp * 16 + h] = v;
+      }
+      ok = named_barrier_and(1, kSoftmaxThreads, local_ok);
+      if (!ok) break;
+      float L[G];
+#pragma unroll
+      for (int h = 0; h < G; ++h) L[h] = (lsum[h] + lsum[16 + h]) + (lsum[32 + h] + lsum[48 + h]);
+
+      const int f = dec::cta_of(item_off, total, P), lst = dec::cta_of(item_off + rows - 1, total, P);
+      bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * kD;
+      if (f == lst) {
+#pragma unroll
+        for (int h = 0; h < G; ++h) outp[h * kD + t] = __float2bfloat16_rn(__uint_as_float(o[h]) / L[h]);
+      } else {
+        float* pbase = dec::partial_slot(a, p, p == f ? 1 : 0, G, kD);
+#pragma unroll
+        for (int h = 0; h < G; ++h) __stcg(pbase + h * kD + t, __uint_as_float(o[h]));
+        float mt = m[0], lt = L[0];
+#pragma unroll
+        for (int h = 1; h < G; ++h) {
+          mt = (t == h) ? m[h] : mt;
+          lt = (t == h) ? L[h] : lt;
+        }
+        if (t < G) {
+          __stcg(pbase + G * kD + t, mt);
+          __stcg(pbase + G * kD + G + t, lt);
+        }
+        dec::merge_item<G, kD, kSoftmaxThreads>(a, p, f, lst, id, outp, ms, sh32 + 1);
+      }
+      named_barrier_sync(1, kSoftmaxThreads);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 5) tmem_dealloc(tmem, kTmemCols);
+  if (threadIdx.x == 0) dec::finish_launch(a);
+}
+
+template <int G>
+cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  decode_tc_kernel<G><<<a.n_ctas, kThreads, SMEM, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool decode_uses_tc(int D, int G) { return D == kD && (G == 7 || G == 8); }
+
+// One CTA per SM; small steps use fewer, at least 512 rows each.
+int decode_tc_ctas(long long total_rows, int num_sms) {
+  const long long by_rows = (total_rows + 511) / 512;
+  long long p = num_sms;
+  if (by_rows < p) p = by_rows;
+  return p < 1 ? 1 : (int)p;
+}
+
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s) {
+  switch (a.geom.G) {
+    case 7: return launch_g<7>(a, s);
+    case 8: return launch_g<8>(a, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace aoh

@@ -36,6 +36,7 @@ struct CacheGeom {
 };
 
 struct DecodeArgs {
+  CUtensorMap tcr, tcs;  // cache regions (see PrefillTcArgs); read by the tcgen05 kernel
   CacheGeom geom;
   const void* q;      // [B][Hq][D]
   const void* k_new;  // [B][Hkv][D]
@@ -66,7 +67,7 @@ struct AppendArgs {
 // Arguments of the tcgen05 prefill kernel: tensor maps over q / k / v
 // ([B][T][H][D], box 128 rows x 64 columns, 128-byte swizzle) and a work list
 // of (b, query head, first row) tiles sorted by cost.
-struct alignas(64) PrefillTcArgs {
+struct PrefillTcArgs {
   CUtensorMap tq, tk, tv;  // the chunk's q / k / v
   CUtensorMap tcr, tcs;    // cache: retrieval / streaming regions as [regions][K, V][rows][D]
   CacheGeom geom;
@@ -85,10 +86,19 @@ void record_error(const char* msg);
 // Launchers (return the launch's cudaError_t).
 bool prefill_tc_make_maps(PrefillTcArgs* a, const void* q, const void* k, const void* v, int B, int T);
 bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv);
+// 4D maps over the retrieval / streaming regions of the cache at `kv`, as
+// [regions][K, V][capacity rows][D] with box [1][1][128][64] and 128-byte
+// swizzle; a kind with no heads leaves its map untouched.
+bool make_cache_region_maps(CUtensorMap* tcr, CUtensorMap* tcs, const CacheGeom& g, const void* kv);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
-// CTAs for a decode launch over `total_rows` cached rows on `num_sms` SMs.
-int decode_ctas(long long total_rows, int num_sms);
+// CTAs for a decode launch over `total_rows` cached rows on `num_sms` SMs
+// (the kernel is chosen by D and G).
+int decode_ctas(long long total_rows, int num_sms, int D, int G);
+// The tcgen05 decode kernel serves (D, G) (else the CUDA-core kernel does).
+bool decode_uses_tc(int D, int G);
+int decode_tc_ctas(long long total_rows, int num_sms);
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
 size_t decode_partial_floats(int n_ctas, int G, int D);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);

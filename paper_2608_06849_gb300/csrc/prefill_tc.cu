@@ -71,20 +71,6 @@ struct PfCfg {
   static_assert(256 + 2 * D <= (int)kTmemCols, "TMEM columns");
 };
 
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_t* err, volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
-      atomicOr(err, kErrTimeout);
-      *abort_flag = 1;
-      return false;
-    }
-  }
-}
-
 // Bits lo..hi-1 of a 32-bit word (lo, hi clamped to [0, 32]).
 __device__ __forceinline__ uint32_t range_bits(int lo, int hi) {
   lo = max(lo, 0);
@@ -572,13 +558,16 @@ static bool make_region_map(CUtensorMap* map, const void* base, int regions, int
   return r == CUDA_SUCCESS;
 }
 
-bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv) {
-  const CacheGeom& g = a->geom;
+bool make_cache_region_maps(CUtensorMap* tcr, CUtensorMap* tcs, const CacheGeom& g, const void* kv) {
   const bf16* base = static_cast<const bf16*>(kv);
   bool ok = true;
-  if (g.n_r > 0) ok = ok && make_region_map(&a->tcr, base + g.r_region(0, 0), g.B * g.n_r, g.max_seq, g.D);
-  if (g.n_s > 0) ok = ok && make_region_map(&a->tcs, base + g.s_region(0, 0), g.B * g.n_s, g.S + g.W, g.D);
+  if (g.n_r > 0) ok = ok && make_region_map(tcr, base + g.r_region(0, 0), g.B * g.n_r, g.max_seq, g.D);
+  if (g.n_s > 0) ok = ok && make_region_map(tcs, base + g.s_region(0, 0), g.B * g.n_s, g.S + g.W, g.D);
   return ok;
+}
+
+bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv) {
+  return make_cache_region_maps(&a->tcr, &a->tcs, a->geom, kv);
 }
 
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s) {

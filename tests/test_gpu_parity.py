@@ -37,6 +37,12 @@ CASES = {
     "mha_group1_d128": (1, 2, 2, 128, 140, 4, 30, [0, 1], None, 3),
     "mha_group1_d64": (2, 3, 3, 64, 90, 0, 7, [1, 0, 1], [90, 41], 3),
     "prefill_multi_tile_ragged": (3, 8, 2, 128, 777, 16, 200, [1, 0], [777, 129, 640], 2),
+    # group sizes 7 and 8 at d 128 decode on the tensor cores: tiles of 128 keys
+    # with tails of 1 and 127 rows, a ring that wraps, several items per CTA
+    "group7_d128_tile_edges": (1, 14, 2, 128, 127, 1, 126, [0, 1], None, 70),
+    "group7_d128_ring_wraps": (1, 7, 1, 128, 40, 3, 5, [1], None, 30),
+    "group8_d128_ragged": (3, 16, 2, 128, 600, 8, 129, [1, 0], [600, 255, 1], 5),
+    "group8_d128_four_heads": (2, 32, 4, 128, 1000, 16, 32, [0, 1, 0, 0], None, 3),
 }
 
 
@@ -59,6 +65,12 @@ def test_long_decode_split_path():
     """Long enough that decode uses many split-KV CTAs and the fused combine."""
     run_case(2, 8, 2, 128, 20000, 64, 1000, [0, 1], decode_steps=3, check_prefill_out=True,
              rows=[0, 1, 63, 64, 1063, 1064, 9999, 19999])
+
+
+def test_long_decode_split_path_group7():
+    """The same at group size 7: each item's rows span more than 16 CTAs, so
+    the split partials merge in two levels."""
+    run_case(2, 14, 2, 128, 20000, 64, 1000, [0, 1], decode_steps=3, check_prefill_out=False)
 
 
 def test_decode_past_capacity_is_refused():

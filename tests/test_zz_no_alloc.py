@@ -22,6 +22,7 @@ pytestmark = pytest.mark.gpu
 @pytest.mark.parametrize("B,Hq,Hkv,D,T,S,W,labels", [
     (4, 32, 8, 128, 9000, 64, 1000, [1, 0, 0, 1, 1, 0, 0, 1]),
     (2, 8, 2, 64, 700, 16, 100, [0, 1]),
+    (2, 28, 4, 128, 5000, 32, 700, [0, 1, 1, 0]),
 ])
 def test_noalloc_decode_matches_handle_decode(B, Hq, Hkv, D, T, S, W, labels):
     ensure_lib()
