@@ -62,7 +62,8 @@ typedef struct aoh_config {
   int32_t batch;      /* B: sequences in the cache, >= 1                           */
   int32_t n_q_heads;  /* Hq, a multiple of n_kv_heads                             */
   int32_t n_kv_heads; /* Hkv                                                      */
-  int32_t d_head;     /* 64 or 128                                                */
+  int32_t d_head;     /* 64 or 128; n_q_heads / n_kv_heads must be 1-8 or 16 for
+                         128, and 1, 2, 4, 7 or 8 for 64 (else UNSUPPORTED)     */
   int32_t max_seq;    /* tokens a retrieval head can hold per sequence, >= 1      */
   int32_t sink;       /* S >= 0: sink tokens kept by a streaming head             */
   int32_t window;     /* W >= 1: recent tokens kept by a streaming head           */

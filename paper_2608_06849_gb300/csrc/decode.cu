@@ -1,6 +1,8 @@
-// Split-KV flash-decode for head-heterogeneous attention (Sec. 5, "Decode
-// Stage", Eq. 8): one new token per sequence; retrieval KV heads attend over
-// their whole history, streaming KV heads over their S sink + W window slots.
+// Split-KV flash-decode for head-heterogeneous attention on CUDA cores (Sec.
+// 5, "Decode Stage", Eq. 8): one new token per sequence; retrieval KV heads
+// attend over their whole history, streaming KV heads over their S sink + W
+// window slots. This kernel serves d_head 64; d_head 128 runs on the tensor
+// cores (decode_tc.cu).
 //
 // One CTA = one (sequence b, KV head, split) work unit; a split is a
 // contiguous range of cache rows. All G query heads of the GQA group are
@@ -401,7 +403,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
           }
         }
       }
-      if (!single) dec::merge_item<G, D, C::NW * 32>(a, p, f, lst, id, outp, mo, sh32 + 1);
+      if (!single) dec::merge_item<G, D, C::NW * 32, false>(a, p, f, lst, id, outp, mo, sh32 + 1);
       named_barrier_sync(1, C::NW * 32);
     }
   }
@@ -427,8 +429,8 @@ cudaError_t launch_cfg(const DecodeArgs& a, cudaStream_t s) {
 }  // namespace
 
 bool decode_supported(int D, int G) {
-  if (D != 64 && D != 128) return false;
-  return G == 1 || G == 2 || G == 4 || G == 7 || G == 8;
+  if (D == 128) return decode_uses_tc(D, G);
+  return D == 64 && (G == 1 || G == 2 || G == 4 || G == 7 || G == 8);
 }
 
 // Two CTAs fit on an SM (about 100 KB of shared memory each), so 2 x SMs
@@ -446,15 +448,7 @@ size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas *
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;
   if (decode_uses_tc(D, G)) return launch_decode_tc(a, s);
-  if (D == 128) {
-    switch (G) {
-      case 1: return launch_cfg<128, 1>(a, s);
-      case 2: return launch_cfg<128, 2>(a, s);
-      case 4: return launch_cfg<128, 4>(a, s);
-      case 7: return launch_cfg<128, 7>(a, s);
-      case 8: return launch_cfg<128, 8>(a, s);
-    }
-  } else if (D == 64) {
+  if (D == 64) {
     switch (G) {
       case 1: return launch_cfg<64, 1>(a, s);
       case 2: return launch_cfg<64, 2>(a, s);

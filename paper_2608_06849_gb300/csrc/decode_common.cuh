@@ -34,26 +34,35 @@ __device__ __forceinline__ int cta_of(long long x, long long total, int P) {
   return (int)(((x + 1) * (long long)P - 1) / total);
 }
 
-// Block-wide prefix sum of the items' rows. On return (after the caller's
-// next __syncthreads) sh64[0] = total rows, sh64[1] = first row of the first
-// item this CTA touches, sh32[0] = that item. `part` is THREADS longs of
-// scratch shared memory.
+// Block-wide prefix sum of the items' rows (warp shuffles, then the warp
+// totals). On return (after the caller's next __syncthreads) sh64[0] = total
+// rows, sh64[1] = first row of the first item this CTA touches, sh32[0] =
+// that item. `wsum` is THREADS / 32 longs of scratch shared memory.
 template <int THREADS>
-__device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* part, long long* sh64, int* sh32) {
+__device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* wsum, long long* sh64, int* sh32) {
+  constexpr int NW = THREADS / 32;
   const CacheGeom& g = a.geom;
   const int n_items = g.B * (g.n_r + g.n_s);
   const int P = a.n_ctas, p = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int per = (n_items + THREADS - 1) / THREADS;
   const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
   long long mine = 0;
   for (int id = i0; id < i1; ++id) mine += item_rows(a, id);
-  part[threadIdx.x] = mine;
+  long long inc = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long y = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) wsum[warp] = inc;
   __syncthreads();
   if (threadIdx.x == 0) {
     long long run = 0;
-    for (int t = 0; t < THREADS; ++t) {
-      const long long v = part[t];
-      part[t] = run;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) {
+      const long long v = wsum[w];
+      wsum[w] = run;
       run += v;
     }
     sh64[0] = run;
@@ -63,7 +72,7 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* p
   __syncthreads();
   const long long total = sh64[0];
   const long long start = (long long)p * total / P;
-  long long off = part[threadIdx.x];
+  long long off = wsum[warp] + inc - mine;
   if (i0 < i1 && off <= start && start < off + mine) {
     int id = i0;
     while (true) {
@@ -88,13 +97,21 @@ __device__ __forceinline__ float* partial_slot(const DecodeArgs& a, int q, int s
 // Merge n partial states (part(j) returns the j-th) with log-sum-exp
 // weights. Writes the normalised bf16 output to `out`, or the merged partial
 // to `dst`. Run by NT threads that share named barrier 1; `scratch` holds
-// n*G + 2*G floats of shared memory.
-template <int G, int D, int NT, class PartFn>
+// 2*n*G + 2*G floats of shared memory. The partials sit in L2; WIDE issues
+// the loads of all of a thread's elements for several parts at once (more
+// registers, fewer round trips).
+template <int G, int D, int NT, bool WIDE, class PartFn>
 __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch) {
-  float* wts = scratch;          // [n][G]
-  float* Ls = scratch + n * G;   // [G]
+  constexpr int E = (G * D + NT - 1) / NT;  // elements per thread
+  float* wts = scratch;          // [n][G] m, then the weights
+  float* ls = scratch + n * G;   // [n][G] l
+  float* Ls = ls + n * G;        // [G]
   float* Ms = Ls + G;            // [G]
-  for (int t = threadIdx.x; t < n * G; t += NT) wts[t] = __ldcg(part(t / G) + G * D + (t % G));
+  for (int t = threadIdx.x; t < n * G; t += NT) {
+    const float* pp = part(t / G) + G * D + (t % G);
+    wts[t] = __ldcg(pp);
+    ls[t] = __ldcg(pp + G);
+  }
   named_barrier_sync(1, NT);
   if (threadIdx.x < G) {
     const int r = threadIdx.x;
@@ -105,17 +122,13 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
       const float mj = wts[j * G + r];
       const float w = (mj == -INFINITY) ? 0.f : fast_exp2(mj - M);
       wts[j * G + r] = w;
-      L += w * __ldcg(part(j) + G * D + G + r);
+      L += w * ls[j * G + r];
     }
     Ls[r] = L;
     Ms[r] = M;
   }
   named_barrier_sync(1, NT);
-  for (int idx = threadIdx.x; idx < G * D; idx += NT) {
-    const int r = idx / D;
-    float O = 0.f;
-#pragma unroll 4
-    for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
+  auto store = [&](int idx, int r, float O) {
     if (out) {
       out[idx] = __float2bfloat16_rn(O / Ls[r]);
     } else {
@@ -124,6 +137,51 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
         __stcg(dst + G * D + r, Ms[r]);
         __stcg(dst + G * D + G + r, Ls[r]);
       }
+    }
+  };
+  if constexpr (!WIDE) {
+    // one element at a time, four parts in flight: few registers
+    for (int idx = threadIdx.x; idx < G * D; idx += NT) {
+      const int r = idx / D;
+      float O = 0.f;
+#pragma unroll 4
+      for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
+      store(idx, r, O);
+    }
+  } else {
+    // every element of the thread at once, U parts in flight
+    constexpr int U = E <= 4 ? 4 : 2;
+    float O[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) O[e] = 0.f;
+    int j = 0;
+    for (; j + U <= n; j += U) {
+      float x[U][E];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const float* pp = part(j + u);
+#pragma unroll
+        for (int e = 0; e < E; ++e) x[u][e] = __ldcg(pp + min((int)threadIdx.x + e * NT, G * D - 1));
+      }
+#pragma unroll
+      for (int e = 0; e < E; ++e) {
+        const int r = min((int)threadIdx.x + e * NT, G * D - 1) / D;
+#pragma unroll
+        for (int u = 0; u < U; ++u) O[e] += wts[(j + u) * G + r] * x[u][e];
+      }
+    }
+    for (; j < n; ++j) {
+      const float* p0 = part(j);
+#pragma unroll
+      for (int e = 0; e < E; ++e) {
+        const int idx = min((int)threadIdx.x + e * NT, G * D - 1);
+        O[e] += wts[j * G + idx / D] * __ldcg(p0 + idx);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const int idx = threadIdx.x + e * NT;
+      if (idx < G * D) store(idx, idx / D, O[e]);
     }
   }
   named_barrier_sync(1, NT);
@@ -136,7 +194,7 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
 // partials and writes the output. A one-group item writes the output at
 // level 1. Run by the NT threads that wrote the partial; `flag` is one int
 // of shared memory, `scratch` as for merge_parts.
-template <int G, int D, int NT>
+template <int G, int D, int NT, bool WIDE>
 __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, int lst, int id,
                                            __nv_bfloat16* outp, float* scratch, volatile int* flag) {
   __threadfence();
@@ -159,10 +217,10 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
     return partial_slot(a, q, q == f ? 1 : 0, G, D);
   };
   if (n_groups == 1) {
-    merge_parts<G, D, NT>(gsz, own, outp, nullptr, scratch);
+    merge_parts<G, D, NT, WIDE>(gsz, own, outp, nullptr, scratch);
     return;
   }
-  merge_parts<G, D, NT>(gsz, own, nullptr, partial_slot(a, p0, 2 + gslot, G, D), scratch);
+  merge_parts<G, D, NT, WIDE>(gsz, own, nullptr, partial_slot(a, p0, 2 + gslot, G, D), scratch);
   __threadfence();
   named_barrier_sync(1, NT);
   if (threadIdx.x == 0) {
@@ -177,7 +235,7 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
     const int q = f + j * kGroup;
     return partial_slot(a, q, 2 + (q == f ? 1 : 0), G, D);
   };
-  merge_parts<G, D, NT>(n_groups, grp_part, outp, nullptr, scratch);
+  merge_parts<G, D, NT, WIDE>(n_groups, grp_part, outp, nullptr, scratch);
 }
 
 // The launch's last CTA advances every sequence length by one. Called by

@@ -1,8 +1,10 @@
-// Split-KV decode on tcgen05 tensor cores for large GQA groups (Sec. 5,
-// "Decode Stage", Eq. 8; d_head = 128). With G query heads per KV head, every
-// cached K/V row meets G queries: 4*G*d flops per 4*d bytes. Above g = 4 that
-// arithmetic no longer hides under the HBM stream on CUDA cores, so here it
-// runs as two skinny MMAs per 128-key tile, with the G heads padded to N = 16:
+// Split-KV decode on tcgen05 tensor cores (Sec. 5, "Decode Stage", Eq. 8;
+// d_head = 128, GQA groups of 1-8 and 16). With G query heads per KV head,
+// every cached K/V row meets G queries: 4*G*d flops per 4*d bytes. On CUDA
+// cores that arithmetic (plus the shuffles that reduce the dot products)
+// stops hiding under the HBM stream above g = 4, and even at g = 4 it costs a
+// few percent; here it runs as two skinny MMAs per 128-key tile, with the G
+// heads padded to N = 16:
 //
 //   S^T[128 keys][16]  = K_tile[128][d] . Q^T           (A = K, K-major; B = Q, K-major)
 //   O^T[d][16]        += V_tile^T[d][128] . P^T[128][16] (A = V, MN-major; B = P, K-major)
@@ -59,7 +61,7 @@ constexpr int OFF_Q = OFF_KV + kNS * kStage;
 constexpr int OFF_P = OFF_Q + 2 * kOpBuf;
 constexpr int OFF_RED = OFF_P + 2 * kOpBuf;   // [2][4][16] warp maxima, [4][16] warp sums
 constexpr int OFF_MS = OFF_RED + (2 * 64 + 64) * 4;
-constexpr int MS_FLOATS = 512;                // merge scratch
+constexpr int MS_FLOATS = 1024;               // merge scratch
 constexpr int OFF_BAR = OFF_MS + MS_FLOATS * 4;
 constexpr int NBAR = 2 * kNS + 2 + 2 + 2 + 2 + 1 + 1;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
@@ -73,7 +75,7 @@ static_assert(kThreads * 8 <= kNS * kStage, "scan scratch");
 template <int G>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
   static_assert(G >= 1 && G <= kN, "group size");
-  static_assert((dec::kGroup + 8) * G + 2 * G <= MS_FLOATS, "merge scratch");
+  static_assert(2 * (dec::kGroup + 8) * G + 2 * G <= MS_FLOATS, "merge scratch");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
   uint8_t* sKV = smem + OFF_KV;
@@ -440,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
           __stcg(pbase + G * kD + t, mt);
           __stcg(pbase + G * kD + G + t, lt);
         }
-        dec::merge_item<G, kD, kSoftmaxThreads>(a, p, f, lst, id, outp, ms, sh32 + 1);
+        dec::merge_item<G, kD, kSoftmaxThreads, true>(a, p, f, lst, id, outp, ms, sh32 + 1);
       }
       named_barrier_sync(1, kSoftmaxThreads);
     }
@@ -467,7 +469,7 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
 
 }  // namespace
 
-bool decode_uses_tc(int D, int G) { return D == kD && (G == 7 || G == 8); }
+bool decode_uses_tc(int D, int G) { return D == kD && ((G >= 1 && G <= 8) || G == 16); }
 
 // One CTA per SM; small steps use fewer, at least 512 rows each.
 int decode_tc_ctas(long long total_rows, int num_sms) {
@@ -479,8 +481,15 @@ int decode_tc_ctas(long long total_rows, int num_sms) {
 
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s) {
   switch (a.geom.G) {
+    case 1: return launch_g<1>(a, s);
+    case 2: return launch_g<2>(a, s);
+    case 3: return launch_g<3>(a, s);
+    case 4: return launch_g<4>(a, s);
+    case 5: return launch_g<5>(a, s);
+    case 6: return launch_g<6>(a, s);
     case 7: return launch_g<7>(a, s);
     case 8: return launch_g<8>(a, s);
+    case 16: return launch_g<16>(a, s);
   }
   return cudaErrorInvalidValue;
 }

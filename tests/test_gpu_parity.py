@@ -43,6 +43,10 @@ CASES = {
     "group7_d128_ring_wraps": (1, 7, 1, 128, 40, 3, 5, [1], None, 30),
     "group8_d128_ragged": (3, 16, 2, 128, 600, 8, 129, [1, 0], [600, 255, 1], 5),
     "group8_d128_four_heads": (2, 32, 4, 128, 1000, 16, 32, [0, 1, 0, 0], None, 3),
+    "group3_d128": (1, 6, 2, 128, 300, 4, 50, [1, 0], None, 3),
+    "group5_d128": (2, 10, 2, 128, 260, 4, 50, [0, 1], [260, 131], 3),
+    "group6_d128": (1, 12, 2, 128, 129, 2, 64, [1, 0], None, 3),
+    "group16_d128": (1, 32, 2, 128, 400, 8, 100, [0, 1], None, 3),
 }
 
 
