@@ -359,8 +359,8 @@ def run_native(args):
                    "hbm_gbs_all_ranks": round(dec_gbs_total, 1),
                    "bytes_per_step": int(avg_bytes), "kernel_us_median": round(statistics.median(per_step_ms) * 1000, 3)},
         "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
-                     "frac": round(dec_gbs / hbm_peak, 4), "traffic": traffic_for("decode"),
-                     "peak_note": f"{peak_note} HBM copy bandwidth; kernel: decode split-KV"},
+                     "frac": round(dec_gbs / hbm_peak, 4), "traffic": traffic_for(decode_kernel_key(wl)),
+                     "peak_note": f"{peak_note} HBM copy bandwidth; kernel: " + decode_kernel_name(wl)},
         "prefill": {"ms": round(pre_ms, 3), "tflops": round(pre_tflops, 2), "flops": flops, "steps": Kp,
                     "tflops_all_ranks": round(pre_tflops_total, 2),
                     "roofline": {"bound": "tensor", "achieved": round(pre_tflops, 2), "peak": tf_peak,
@@ -376,6 +376,19 @@ def run_native(args):
         "cpu_baseline": cpu,
     }
     print(json.dumps(line))
+
+
+def decode_kernel_key(wl):
+    """Which decode kernel serves this shape (the library's dispatch: d_head
+    128 runs on the tensor cores, d_head 64 on CUDA cores)."""
+    return "decode_tc" if wl.d_head == 128 else "decode"
+
+
+def decode_kernel_name(wl):
+    g = wl.n_q_heads // wl.n_kv_heads
+    if wl.d_head == 128:
+        return f"decode_tc_kernel<{g}> (tcgen05 split-KV)"
+    return f"decode_kernel<DecodeCfg<64,{g}>> (CUDA-core split-KV)"
 
 
 def traffic_for(kernel):
