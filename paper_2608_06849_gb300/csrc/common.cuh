@@ -105,6 +105,12 @@ __device__ __forceinline__ void named_barrier_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Release / acquire fence at GPU scope (lighter than the sequentially
+// consistent __threadfence). After a CTA barrier, one thread's fence orders
+// the whole CTA's earlier stores before its next relaxed atomic (release),
+// or that atomic before the CTA's later loads (acquire).
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+
 // Named barrier over `count` threads that also returns the AND of `pred`
 // over them (every thread of the barrier gets the same answer).
 __device__ __forceinline__ bool named_barrier_and(int id, int count, bool pred) {

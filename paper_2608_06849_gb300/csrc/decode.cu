@@ -443,7 +443,7 @@ int decode_ctas(long long total_rows, int num_sms, int D, int G) {
   return p < 1 ? 1 : (int)p;
 }
 
-size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 4 * G * (D + 2); }
+size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 4 * dec::partial_stride(G, D); }
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;

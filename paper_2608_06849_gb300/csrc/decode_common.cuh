@@ -87,101 +87,138 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* w
 }
 
 // Partial state of split CTA q for an item whose first CTA is f: o[G][D]
-// (unnormalised), then m[G] (running max, log2 units), then l[G]. Slot 0/1:
-// the CTA's first / last shared item; slot 2/3: the group partial of the
-// group the CTA heads.
+// (unnormalised), then m[G] (running max, log2 units), then l[G], in slots
+// of partial_stride floats (16-byte aligned). Slot 0/1: the CTA's first /
+// last shared item; slot 2/3: the group partial of the group the CTA heads.
+__host__ __device__ constexpr int partial_stride(int G, int D) { return (G * (D + 2) + 3) / 4 * 4; }
+
 __device__ __forceinline__ float* partial_slot(const DecodeArgs& a, int q, int slot, int G, int D) {
-  return a.partials + ((size_t)q * 4 + slot) * (size_t)(G * (D + 2));
+  return a.partials + ((size_t)q * 4 + slot) * (size_t)partial_stride(G, D);
 }
 
 // Merge n partial states (part(j) returns the j-th) with log-sum-exp
 // weights. Writes the normalised bf16 output to `out`, or the merged partial
-// to `dst`. Run by NT threads that share named barrier 1; `scratch` holds
-// 2*n*G + 2*G floats of shared memory. The partials sit in L2; WIDE issues
-// the loads of all of a thread's elements for several parts at once (more
-// registers, fewer round trips).
+// to `dst`. Run by NT threads that share named barrier 1. The partials sit
+// in L2, so the merge is a chain of L2 round trips at the end of the launch.
+//
+// WIDE = false (few registers): m and l are staged in `scratch` (2*n*G + 2*G
+// floats of shared memory), then each thread sums one element at a time.
+// WIDE = true: each thread owns E4 float4 groups of elements; every batch of
+// U parts costs one round trip (O, m and l of all U parts loaded together)
+// and folds into a running per-element max, as in the online softmax.
 template <int G, int D, int NT, bool WIDE, class PartFn>
 __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch) {
-  constexpr int E = (G * D + NT - 1) / NT;  // elements per thread
-  float* wts = scratch;          // [n][G] m, then the weights
-  float* ls = scratch + n * G;   // [n][G] l
-  float* Ls = ls + n * G;        // [G]
-  float* Ms = Ls + G;            // [G]
-  for (int t = threadIdx.x; t < n * G; t += NT) {
-    const float* pp = part(t / G) + G * D + (t % G);
-    wts[t] = __ldcg(pp);
-    ls[t] = __ldcg(pp + G);
-  }
-  named_barrier_sync(1, NT);
-  if (threadIdx.x < G) {
-    const int r = threadIdx.x;
-    float M = -INFINITY;
-    for (int j = 0; j < n; ++j) M = fmaxf(M, wts[j * G + r]);
-    float L = 0.f;
-    for (int j = 0; j < n; ++j) {
-      const float mj = wts[j * G + r];
-      const float w = (mj == -INFINITY) ? 0.f : fast_exp2(mj - M);
-      wts[j * G + r] = w;
-      L += w * ls[j * G + r];
-    }
-    Ls[r] = L;
-    Ms[r] = M;
-  }
-  named_barrier_sync(1, NT);
-  auto store = [&](int idx, int r, float O) {
-    if (out) {
-      out[idx] = __float2bfloat16_rn(O / Ls[r]);
-    } else {
-      __stcg(dst + idx, O);
-      if (idx - r * D == 0) {
-        __stcg(dst + G * D + r, Ms[r]);
-        __stcg(dst + G * D + G + r, Ls[r]);
-      }
-    }
-  };
   if constexpr (!WIDE) {
-    // one element at a time, four parts in flight: few registers
+    float* wts = scratch;          // [n][G] m, then the weights
+    float* ls = scratch + n * G;   // [n][G] l
+    float* Ls = ls + n * G;        // [G]
+    float* Ms = Ls + G;            // [G]
+    for (int t = threadIdx.x; t < n * G; t += NT) {
+      const float* pp = part(t / G) + G * D + (t % G);
+      wts[t] = __ldcg(pp);
+      ls[t] = __ldcg(pp + G);
+    }
+    named_barrier_sync(1, NT);
+    if (threadIdx.x < G) {
+      const int r = threadIdx.x;
+      float M = -INFINITY;
+      for (int j = 0; j < n; ++j) M = fmaxf(M, wts[j * G + r]);
+      float L = 0.f;
+      for (int j = 0; j < n; ++j) {
+        const float mj = wts[j * G + r];
+        const float w = (mj == -INFINITY) ? 0.f : fast_exp2(mj - M);
+        wts[j * G + r] = w;
+        L += w * ls[j * G + r];
+      }
+      Ls[r] = L;
+      Ms[r] = M;
+    }
+    named_barrier_sync(1, NT);
     for (int idx = threadIdx.x; idx < G * D; idx += NT) {
       const int r = idx / D;
       float O = 0.f;
 #pragma unroll 4
       for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
-      store(idx, r, O);
+      if (out) {
+        out[idx] = __float2bfloat16_rn(O / Ls[r]);
+      } else {
+        __stcg(dst + idx, O);
+        if (idx - r * D == 0) {
+          __stcg(dst + G * D + r, Ms[r]);
+          __stcg(dst + G * D + G + r, Ls[r]);
+        }
+      }
     }
   } else {
-    // every element of the thread at once, U parts in flight
-    constexpr int U = E <= 4 ? 4 : 2;
-    float O[E];
+    constexpr int NV = G * D / 4;
+    constexpr int E4 = (NV + NT - 1) / NT;
+    constexpr int U = E4 <= 2 ? 8 : 4;
+    float4 O[E4];
+    float M[E4], L[E4];
+    int vv[E4], rr[E4];
 #pragma unroll
-    for (int e = 0; e < E; ++e) O[e] = 0.f;
-    int j = 0;
-    for (; j + U <= n; j += U) {
-      float x[U][E];
+    for (int e = 0; e < E4; ++e) {
+      O[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+      M[e] = -INFINITY;
+      L[e] = 0.f;
+      vv[e] = min((int)threadIdx.x + e * NT, NV - 1);
+      rr[e] = vv[e] * 4 / D;
+    }
+    for (int j = 0; j < n; j += U) {
+      float4 x[U][E4];
+      float mj[U][E4], lj[U][E4];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const float* pp = part(j + u);
+        const float* pp = part(min(j + u, n - 1));
 #pragma unroll
-        for (int e = 0; e < E; ++e) x[u][e] = __ldcg(pp + min((int)threadIdx.x + e * NT, G * D - 1));
+        for (int e = 0; e < E4; ++e) {
+          x[u][e] = __ldcg(reinterpret_cast<const float4*>(pp) + vv[e]);
+          mj[u][e] = __ldcg(pp + G * D + rr[e]);
+          lj[u][e] = __ldcg(pp + G * D + G + rr[e]);
+        }
       }
 #pragma unroll
-      for (int e = 0; e < E; ++e) {
-        const int r = min((int)threadIdx.x + e * NT, G * D - 1) / D;
+      for (int e = 0; e < E4; ++e) {
+        float bm = M[e];
 #pragma unroll
-        for (int u = 0; u < U; ++u) O[e] += wts[(j + u) * G + r] * x[u][e];
+        for (int u = 0; u < U; ++u)
+          if (j + u < n) bm = fmaxf(bm, mj[u][e]);
+        const float sc = (M[e] == -INFINITY) ? 0.f : fast_exp2(M[e] - bm);
+        O[e].x *= sc;
+        O[e].y *= sc;
+        O[e].z *= sc;
+        O[e].w *= sc;
+        L[e] *= sc;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const float w = (j + u < n && mj[u][e] != -INFINITY) ? fast_exp2(mj[u][e] - bm) : 0.f;
+          O[e].x += w * x[u][e].x;
+          O[e].y += w * x[u][e].y;
+          O[e].z += w * x[u][e].z;
+          O[e].w += w * x[u][e].w;
+          L[e] += w * lj[u][e];
+        }
+        M[e] = bm;
       }
     }
-    for (; j < n; ++j) {
-      const float* p0 = part(j);
 #pragma unroll
-      for (int e = 0; e < E; ++e) {
-        const int idx = min((int)threadIdx.x + e * NT, G * D - 1);
-        O[e] += wts[j * G + idx / D] * __ldcg(p0 + idx);
+    for (int e = 0; e < E4; ++e) {
+      const int v = threadIdx.x + e * NT;
+      if (v >= NV) break;
+      const int idx = v * 4, r = rr[e];
+      if (out) {
+        const float inv = 1.f / L[e];
+        uint2 w;
+        w.x = float2_to_bf16x2(O[e].x * inv, O[e].y * inv);
+        w.y = float2_to_bf16x2(O[e].z * inv, O[e].w * inv);
+        *reinterpret_cast<uint2*>(out + idx) = w;
+      } else {
+        __stcg(reinterpret_cast<float4*>(dst + idx), O[e]);
+        if (idx - r * D == 0) {
+          __stcg(dst + G * D + r, M[e]);
+          __stcg(dst + G * D + G + r, L[e]);
+        }
       }
-    }
-#pragma unroll
-    for (int e = 0; e < E; ++e) {
-      const int idx = threadIdx.x + e * NT;
-      if (idx < G * D) store(idx, idx / D, O[e]);
     }
   }
   named_barrier_sync(1, NT);
@@ -197,7 +234,9 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
 template <int G, int D, int NT, bool WIDE>
 __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, int lst, int id,
                                            __nv_bfloat16* outp, float* scratch, volatile int* flag) {
-  __threadfence();
+  // the barrier orders every thread's partial stores before thread 0's fence
+  // and counter update (release); thread 0's fence after a last arrival
+  // orders the other parts' stores before the loads below (acquire)
   named_barrier_sync(1, NT);
   const int np = lst - f + 1;
   const int gi = (p - f) / kGroup, p0 = f + gi * kGroup;
@@ -205,13 +244,17 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
   const int n_groups = (np + kGroup - 1) / kGroup;
   const int gslot = (p0 == f) ? 1 : 0;  // the item is p0's last item iff p0 == f
   if (threadIdx.x == 0) {
+    fence_acq_rel_gpu();
     const uint32_t prev = atomicAdd(&a.gcounters[p0 * 2 + gslot], 1u);
-    *flag = (prev == (uint32_t)(gsz - 1));
+    const bool last = prev == (uint32_t)(gsz - 1);
+    if (last) {
+      fence_acq_rel_gpu();
+      a.gcounters[p0 * 2 + gslot] = 0u;
+    }
+    *flag = last;
   }
   named_barrier_sync(1, NT);
   if (!*flag) return;
-  __threadfence();
-  if (threadIdx.x == 0) a.gcounters[p0 * 2 + gslot] = 0u;
   auto own = [&](int j) {
     const int q = p0 + j;
     return partial_slot(a, q, q == f ? 1 : 0, G, D);
@@ -221,16 +264,18 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
     return;
   }
   merge_parts<G, D, NT, WIDE>(gsz, own, nullptr, partial_slot(a, p0, 2 + gslot, G, D), scratch);
-  __threadfence();
-  named_barrier_sync(1, NT);
   if (threadIdx.x == 0) {
+    fence_acq_rel_gpu();
     const uint32_t prev = atomicAdd(&a.counters[id], 1u);
-    *flag = (prev == (uint32_t)(n_groups - 1));
+    const bool last = prev == (uint32_t)(n_groups - 1);
+    if (last) {
+      fence_acq_rel_gpu();
+      a.counters[id] = 0u;
+    }
+    *flag = last;
   }
   named_barrier_sync(1, NT);
   if (!*flag) return;
-  __threadfence();
-  if (threadIdx.x == 0) a.counters[id] = 0u;
   auto grp_part = [&](int j) {
     const int q = f + j * kGroup;
     return partial_slot(a, q, 2 + (q == f ? 1 : 0), G, D);

@@ -103,7 +103,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   const int n_items = g.B * HK;
   const int P = a.n_ctas, p = blockIdx.x;
 
-  dec::find_cta_range<kThreads>(a, reinterpret_cast<long long*>(sKV), sh64, sh32);
+  // Prologue that touches no global memory; it may overlap the tail of the
+  // previous kernel on the stream (programmatic dependent launch).
   // Q and P rows >= G stay zero for the whole launch
   for (int i = threadIdx.x; i < 4 * kOpBuf / 16; i += kThreads)
     reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0, 0, 0, 0);
@@ -132,6 +133,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // everything the previous kernels wrote (lengths, cache, inputs, counters)
+  // is visible after this wait; the next step may then start its prologue
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  dec::find_cta_range<kThreads>(a, reinterpret_cast<long long*>(sKV), sh64, sh32);
+  __syncthreads();
   const long long total = sh64[0];
   const long long start = (long long)p * total / P;
   const long long end = (long long)(p + 1) * total / P;
@@ -463,8 +470,19 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  decode_tc_kernel<G><<<a.n_ctas, kThreads, SMEM, s>>>(a);
-  return cudaGetLastError();
+  // programmatic stream serialization: the kernel waits for the previous
+  // work on the stream itself (griddepcontrol.wait) after its prologue
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.n_ctas);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<G>, a);
 }
 
 }  // namespace
