@@ -18,9 +18,14 @@ Stage"; Appendix "GQA Extension"):
 Readings taken where the paper is silent (each one is listed in the design doc):
   * the recent window counts the query's own position, so a streaming query
     at position i sees key j iff ``j <= i and (j < S or i - j < W)``;
-  * prefill uses that per-token rule for every row (a chunk size of one),
-    which makes prefill row t and a decode step at position t the same
-    computation;
+  * prefill uses that per-token rule for every row by default, which makes
+    prefill row t and a decode step at position t the same computation;
+  * the literal chunk rule of the "Chunked-Prefill Stage" (evict all but the
+    sinks and the W most recent tokens after each chunk of K tokens) is the
+    ``chunk=K`` option of the prefill functions: a streaming query at
+    position i in chunk c = i // K sees key j iff ``j <= i and (j < S or
+    j >= c*K - W)`` (the cache as it stood after chunk c - 1, plus chunk c
+    itself). Decode keeps the per-token rule in both modes;
   * query head h belongs to KV head ``h // (Hq // Hkv)``;
   * the score scale is ``1/sqrt(d_head)``.
 """
@@ -31,26 +36,32 @@ RETRIEVAL = 0
 STREAMING = 1
 
 
-def allowed(i, j, streaming, S, W):
-    """True iff query position i may attend key position j (scalar form)."""
+def allowed(i, j, streaming, S, W, chunk=0):
+    """True iff query position i may attend key position j (scalar form).
+    chunk = 0: the per-token window; chunk = K > 0: eviction after each
+    K-token chunk (see the module docstring)."""
     if j > i:
         return False
     if not streaming:
         return True
+    if chunk:
+        return j < S or j >= (i // chunk) * chunk - W
     return j < S or i - j < W
 
 
-def allowed_mask(q_pos, k_pos, streaming, S, W):
+def allowed_mask(q_pos, k_pos, streaming, S, W, chunk=0):
     """Boolean [len(q_pos), len(k_pos)] mask; the vector form of ``allowed``."""
     i = np.asarray(q_pos, dtype=np.int64)[:, None]
     j = np.asarray(k_pos, dtype=np.int64)[None, :]
     causal = j <= i
     if not streaming:
         return causal
+    if chunk:
+        return causal & ((j < S) | (j >= (i // chunk) * chunk - W))
     return causal & ((j < S) | (i - j < W))
 
 
-def attend(q_rows, q_pos, k, v, labels, S, W):
+def attend(q_rows, q_pos, k, v, labels, S, W, chunk=0):
     """Attention output for a set of query rows of one sequence.
 
     q_rows  [R, Hq, d]   queries, float64
@@ -79,7 +90,7 @@ def attend(q_rows, q_pos, k, v, labels, S, W):
     scale = 1.0 / np.sqrt(d)
     for kv in range(Hkv):
         streaming = int(labels[kv]) == STREAMING
-        mask = allowed_mask(q_pos, k_pos, streaming, S, W)
+        mask = allowed_mask(q_pos, k_pos, streaming, S, W, chunk)
         for h in range(kv * g, (kv + 1) * g):
             s = (q_rows[:, h, :] @ k[:, kv, :].T) * scale
             s = np.where(mask, s, -np.inf)
@@ -90,16 +101,18 @@ def attend(q_rows, q_pos, k, v, labels, S, W):
     return out
 
 
-def prefill(q, k, v, labels, S, W, rows=None):
+def prefill(q, k, v, labels, S, W, rows=None, chunk=0):
     """Prefill output of one sequence: rows of ``attend`` over its own keys.
 
     q [T, Hq, d], k/v [T, Hkv, d]. ``rows`` selects the query positions to
     compute (all T when None); every row only ever sees keys at positions
     <= itself, so any subset is computed exactly as in the full matrix.
+    ``chunk``: 0 for the per-token streaming window, K > 0 for eviction
+    after each K-token chunk.
     """
     T = q.shape[0]
     rows = np.arange(T) if rows is None else np.asarray(rows, dtype=np.int64)
-    return attend(np.asarray(q)[rows], rows, k, v, labels, S, W)
+    return attend(np.asarray(q)[rows], rows, k, v, labels, S, W, chunk)
 
 
 def decode_step(q_new, k_seq, v_seq, labels, S, W):

@@ -8,7 +8,11 @@ the module disagrees with what the paper and the mathematics fix:
   * closed forms: S=0, W=1 returns V itself; S=1, W=1 is a two-key softmax;
   * invariants: a window that covers the whole sequence equals retrieval;
     a decode step equals the matching prefill row;
-  * the ring-buffer slot model holds exactly the attended positions.
+  * the ring-buffer slot model holds exactly the attended positions;
+  * the chunk-eviction option against a step-by-step simulation of the
+    procedure of the "Chunked-Prefill Stage" (process a chunk against the
+    cache, then evict all but the sinks and the W most recent tokens), plus
+    two closed forms (chunks of one token; one chunk covering the prompt).
 """
 
 import math
@@ -185,6 +189,67 @@ def pin_ring_slot_layout(att):
                 slot = S if slot == S + W - 1 else slot + 1
 
 
+def chunked_prefill_simulation(q, k, v, labels, S, W, K):
+    """The chunked-prefill procedure run step by step for streaming heads:
+    chunk c's queries attend to the cached positions plus the chunk's own
+    positions up to themselves; after the chunk every cached position except
+    the S sinks and the W most recent is evicted. Retrieval heads keep all."""
+    T, Hq, d = q.shape
+    Hkv = k.shape[1]
+    g = Hq // Hkv
+    out = np.zeros_like(q)
+    for kv in range(Hkv):
+        cache = []                       # positions held before the current chunk
+        for c0 in range(0, T, K):
+            chunk = list(range(c0, min(c0 + K, T)))
+            for i in chunk:
+                keys = cache + [j for j in chunk if j <= i]
+                if labels[kv] == 0:
+                    keys = list(range(i + 1))
+                for h in range(kv * g, (kv + 1) * g):
+                    sc = np.array([q[i, h] @ k[j, kv] for j in keys]) / math.sqrt(d)
+                    w = np.exp(sc - sc.max())
+                    out[i, h] = (w[:, None] * v[keys, kv]).sum(axis=0) / w.sum()
+            held = cache + chunk
+            recent = sorted(p for p in held if p >= S)[-W:] if W > 0 else []
+            cache = [p for p in held if p < S] + recent
+    return out
+
+
+def pin_chunk_eviction_simulation(att):
+    rng = _rng(8)
+    cases = [
+        (30, 4, 2, 8, [1, 0], 2, 5, 7),
+        (41, 2, 1, 8, [1], 0, 3, 4),
+        (25, 4, 2, 4, [1, 1], 3, 2, 10),
+        (20, 2, 1, 8, [1], 1, 1, 1),
+        (33, 4, 2, 8, [0, 1], 4, 6, 40),
+    ]
+    for T, Hq, Hkv, d, labels, S, W, K in cases:
+        q, k, v = _qkv(rng, T, Hq, Hkv, d, peaky=2.0)
+        got = att.prefill(q, k, v, labels, S, W, chunk=K)
+        want = chunked_prefill_simulation(q, k, v, labels, S, W, K)
+        np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+
+
+def pin_chunk_closed_forms(att):
+    """Chunks of one token see the sinks plus the W positions before the
+    query and the query itself: the per-token rule with a window of W + 1.
+    One chunk covering the prompt sees everything causally (retrieval)."""
+    rng = _rng(9)
+    T, Hq, Hkv, d = 29, 4, 2, 8
+    q, k, v = _qkv(rng, T, Hq, Hkv, d, peaky=2.0)
+    for S, W in [(0, 1), (2, 4), (3, 9)]:
+        a = att.prefill(q, k, v, [1, 0], S, W, chunk=1)
+        b = att.prefill(q, k, v, [1, 0], S, W + 1)
+        np.testing.assert_array_equal(a, b)
+        a = att.prefill(q, k, v, [1, 1], S, W, chunk=T)
+        b = att.prefill(q, k, v, [0, 0], S, W)
+        np.testing.assert_array_equal(a, b)
+    # chunk = 0 is the per-token rule
+    np.testing.assert_array_equal(att.prefill(q, k, v, [1, 0], 2, 4, chunk=0), att.prefill(q, k, v, [1, 0], 2, 4))
+
+
 ALL_PINS = [
     pin_brute_force,
     pin_library_sdpa,
@@ -194,4 +259,6 @@ ALL_PINS = [
     pin_decode_is_prefill_row,
     pin_ring_holds_attended_set,
     pin_ring_slot_layout,
+    pin_chunk_eviction_simulation,
+    pin_chunk_closed_forms,
 ]

@@ -28,6 +28,9 @@ MUTANTS = {
     "ring_slot_wrong_base": ("return S + (p - S) % W", "return S + p % W"),
     "value_uses_key": ("out[:, h, :] = p @ v[:, kv, :]", "out[:, h, :] = p @ k[:, kv, :]"),
     "decode_wrong_row": ("t = k_seq.shape[0] - 1", "t = k_seq.shape[0] - 2"),
+    "chunk_window_off_by_one": ("(j >= (i // chunk) * chunk - W))", "(j > (i // chunk) * chunk - W))"),
+    "chunk_per_query": ("(j >= (i // chunk) * chunk - W))", "(j >= i - W))"),
+    "chunk_ignored": ("    if chunk:\n        return causal", "    if False:\n        return causal"),
 }
 
 
