@@ -21,7 +21,9 @@
  *   - Query head h belongs to KV head h / (n_q_heads / n_kv_heads).
  *   - A key at position j is visible to the query at position i iff j <= i
  *     and, for a streaming KV head, (j < S or i - j < W): the window counts
- *     the query's own position.
+ *     the query's own position (aoh_config.chunk = 0, and every decode step).
+ *     With aoh_config.chunk = K > 0, prefill rows of a streaming head use
+ *     the chunk-eviction rule documented at that field.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream). Calls are asynchronous and stream-ordered; calls that use one
  *     cache must be ordered on one stream (or synchronised by the caller).
@@ -67,6 +69,11 @@ typedef struct aoh_config {
   int32_t max_seq;    /* tokens a retrieval head can hold per sequence, >= 1      */
   int32_t sink;       /* S >= 0: sink tokens kept by a streaming head             */
   int32_t window;     /* W >= 1: recent tokens kept by a streaming head           */
+  int32_t chunk;      /* streaming prefill rule: 0 = per-token window (below);
+                         K >= 1 = eviction after each K-token chunk (Sec. 5,
+                         "Chunked-Prefill Stage"): a prefill row at position i
+                         of chunk c = i / K sees keys j <= i with j < S or
+                         j >= c*K - W. Decode always uses the per-token rule. */
 } aoh_config;
 
 typedef struct aoh_cache aoh_cache; /* opaque handle */
@@ -117,6 +124,9 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
  *   q    [B][T][n_q_heads][d_head]
  *   k, v [B][T][n_kv_heads][d_head]
  *   T    padded chunk length, >= 1.
+ * With aoh_config.chunk = K > 0, every L_b must be a multiple of K (a call
+ * starts on a chunk boundary; INVALID otherwise); a call may span several
+ * chunks.
  *   seq_lens  host array [B] of chunk lengths 1..T, or NULL (all T). Rows at
  *             or past seq_lens[b] are ignored: their contents (even NaN) do
  *             not affect any output, and their outputs are not written.
@@ -215,7 +225,7 @@ aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_la
                                    int32_t* lens, int32_t max_len, const void* q, const void* k_new,
                                    const void* v_new, void* out, void* stream);
 
-/* Library ABI version (major * 100 + minor). */
+/* Library ABI version (major * 100 + minor); 101 added aoh_config.chunk. */
 int32_t aoh_version(void);
 
 #ifdef __cplusplus

@@ -46,7 +46,7 @@ class AohError(RuntimeError):
 
 class aoh_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
-                ("batch", "n_q_heads", "n_kv_heads", "d_head", "max_seq", "sink", "window")]
+                ("batch", "n_q_heads", "n_kv_heads", "d_head", "max_seq", "sink", "window", "chunk")]
 
 
 _lib = None
@@ -97,8 +97,10 @@ def _labels_arr(labels):
     return (ctypes.c_uint8 * len(labels))(*[int(x) for x in labels])
 
 
-def make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window):
-    return aoh_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window)
+def make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, chunk=0):
+    """chunk = 0: per-token streaming window; K > 0: streaming prefill rows
+    evict after each K-token chunk (aoh_config.chunk)."""
+    return aoh_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, chunk)
 
 
 def _stream_ptr(stream):
@@ -188,14 +190,14 @@ def aoh_cache_destroy(cache):
 class Cache:
     """A KV buffer on the current CUDA device plus its library handle."""
 
-    def __init__(self, batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, labels, device=None):
-        self.cfg = make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window)
+    def __init__(self, batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, labels, device=None, chunk=0):
+        self.cfg = make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, chunk)
         self.labels = [int(x) for x in labels]
         self.nbytes = aoh_cache_bytes(self.cfg, self.labels)
         self.buffer = torch.empty(self.nbytes, dtype=torch.uint8, device=device or "cuda")
         self.handle = aoh_cache_init(self.cfg, self.labels, self.buffer)
         self.batch, self.n_q_heads, self.n_kv_heads, self.d_head = batch, n_q_heads, n_kv_heads, d_head
-        self.max_seq, self.sink, self.window = max_seq, sink, window
+        self.max_seq, self.sink, self.window, self.chunk = max_seq, sink, window, chunk
 
     def prefill(self, q, k, v, out=None, seq_lens=None, stream=None):
         aoh_prefill(q, k, v, k.shape[1], seq_lens, self.handle, out, stream)

@@ -46,6 +46,7 @@ aoh_status check_config(const aoh_config* cfg, const uint8_t* labels, int* n_r, 
   if (c.n_q_heads % c.n_kv_heads) return fail(AOH_ERR_INVALID, "n_q_heads must be a multiple of n_kv_heads");
   if (c.d_head != 64 && c.d_head != 128) return fail(AOH_ERR_UNSUPPORTED, "d_head must be 64 or 128");
   if (c.sink < 0 || c.window < 1) return fail(AOH_ERR_INVALID, "need sink >= 0 and window >= 1");
+  if (c.chunk < 0) return fail(AOH_ERR_INVALID, "chunk must be >= 0");
   int r = 0, s = 0;
   for (int h = 0; h < c.n_kv_heads; ++h) {
     if (labels[h] == AOH_RETRIEVAL)
@@ -81,7 +82,7 @@ std::vector<int4> prefill_schedule(const CacheGeom& g, const std::vector<int32_t
           n = (q_end + BN - 1) / BN;
         } else {
           const int a_end = (std::min(std::max(S_rel, 0), q_end) + BN - 1) / BN;
-          const int c_begin = std::max(a_end, std::max(0, q0 - g.W + 1) / BN);
+          const int c_begin = std::max(a_end, std::max(0, g.wstart(q0)) / BN);
           const int c_end = std::max(c_begin, (q_end + BN - 1) / BN);
           n = a_end + (c_end - c_begin);
         }
@@ -128,7 +129,7 @@ struct aoh_cache {
 
 extern "C" {
 
-int32_t aoh_version(void) { return 100; }
+int32_t aoh_version(void) { return 101; }
 
 const char* aoh_last_error(void) { return g_last_error.c_str(); }
 
@@ -170,6 +171,7 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   g.max_seq = c.max_seq;
   g.S = c.sink;
   g.W = c.window;
+  g.K = c.chunk;
   g.n_r = n_r;
   g.n_s = n_s;
   int ir = 0, is = 0;
@@ -286,6 +288,10 @@ aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, c
     }
   }
   const std::vector<int32_t> base = cache->lens;
+  if (g.K > 0)
+    for (int b = 0; b < g.B; ++b)
+      if (base[b] % g.K)
+        return fail(AOH_ERR_INVALID, "sequence %d holds %d tokens, not a multiple of chunk %d", b, base[b], g.K);
   std::vector<int32_t> lens(g.B);
   bool chunked = false;
   for (int b = 0; b < g.B; ++b) {

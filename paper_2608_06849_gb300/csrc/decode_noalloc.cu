@@ -80,6 +80,7 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   g.max_seq = c.max_seq;
   g.S = c.sink;
   g.W = c.window;
+  g.K = c.chunk;
   int n_r = 0, n_s = 0;
   for (int h = 0; h < c.n_kv_heads; ++h) {
     if (head_labels[h] == AOH_RETRIEVAL) {

@@ -15,6 +15,7 @@ constexpr int kMaxKvHeads = 64;
 struct CacheGeom {
   int B, Hq, Hkv, D, G;
   int max_seq, S, W;
+  int K;  // streaming prefill eviction chunk; 0 = per-token window
   int n_r, n_s;
   // kind[h] = 0 retrieval / 1 streaming; idx[h] = index among heads of its kind
   uint8_t kind[kMaxKvHeads];
@@ -33,6 +34,12 @@ struct CacheGeom {
     return kind[h] ? s_region(b, idx[h]) : r_region(b, idx[h]);
   }
   __host__ __device__ int capacity(int h) const { return kind[h] ? S + W : max_seq; }
+  // First non-sink key a streaming prefill row may see, for row i counted
+  // from the start of the prefill call (calls start on chunk boundaries when
+  // K > 0): the per-token window i - W + 1, or, with eviction after each
+  // K-token chunk, the W positions before the row's chunk (Sec. 5,
+  // "Chunked-Prefill Stage").
+  __host__ __device__ int wstart(int i) const { return K ? (i / K) * K - W : i - W + 1; }
 };
 
 struct DecodeArgs {

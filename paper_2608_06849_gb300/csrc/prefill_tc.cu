@@ -121,7 +121,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
     c_begin = c_end = a_end;
   } else {
     a_end = (min(max(S_rel, 0), q_end) + kBN - 1) / kBN;
-    c_begin = max(a_end, max(0, q0 - g.W + 1) / kBN);
+    c_begin = max(a_end, max(0, g.wstart(q0)) / kBN);
     c_end = max(c_begin, (q_end + kBN - 1) / kBN);
   }
   const int n_tiles = n_c + a_end + (c_end - c_begin);
@@ -357,11 +357,13 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
         } else {
           need_mask = true;
           e_hi = min(S, Lb) - j0;
+          // cached positions the row may see: sinks, and [Lb + wstart(i), Lb)
+          const int skip = W + g.wstart(i);  // oldest ring positions hidden
           if (Lb <= S + W) {
-            a0 = max(S, Lb + i - W + 1) - j0;
+            a0 = max(S, Lb + g.wstart(i)) - j0;
             a1 = Lb - j0;
-          } else if (i + 1 < W) {
-            const int u = rot + i + 1;
+          } else if (skip < W) {
+            const int u = rot + max(skip, 0);
             if (u < W) {
               a0 = S + u - j0;
               a1 = S + W - j0;
@@ -375,13 +377,13 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
         }
       } else {
         const int jl = j0 + kBN - 1;
-        need_mask = !(jl <= qx0 && jl < len && (!streaming || jl < S_rel || (qx0 + kBM - 1) - j0 < W));
+        need_mask = !(jl <= qx0 && jl < len && (!streaming || jl < S_rel || j0 >= g.wstart(qx0 + kBM - 1)));
         const int kmax = min(i, len - 1) - j0;
         if (!streaming) {
           e_hi = kmax + 1;
         } else {
           e_hi = min(kmax + 1, S_rel - j0);
-          a0 = i - W + 1 - j0;
+          a0 = g.wstart(i) - j0;
           a1 = kmax + 1;
         }
       }

@@ -55,7 +55,7 @@ def test_noalloc_rejects_bad_arguments_on_host(lib):
 
 
 def test_version(lib):
-    assert aoh.aoh_version() == 100
+    assert aoh.aoh_version() == 101
 
 
 @pytest.mark.parametrize("B,Hq,Hkv,d,max_seq,S,W,labels", [
@@ -92,6 +92,22 @@ def test_invalid_config_rejected_on_host(lib, bad):
     n = lib.aoh_cache_bytes(ctypes.byref(cfg), (ctypes.c_uint8 * 4)(0, 1, 0, 1))
     assert n == 0
     assert lib.aoh_last_error().decode() != ""
+
+
+def test_negative_chunk_rejected(lib):
+    cfg = aoh.make_config(1, 8, 2, 64, 64, 4, 8, chunk=-1)
+    assert lib.aoh_cache_bytes(ctypes.byref(cfg), (ctypes.c_uint8 * 2)(0, 1)) == 0
+    assert "chunk" in lib.aoh_last_error().decode()
+
+
+def test_config_struct_matches_header():
+    """aoh_config is eight int32 fields, in the header's order."""
+    import re
+    hdr = open(os.path.join(ROOT, "include", "aoh.h")).read()
+    body = re.search(r"typedef struct aoh_config \{(.*?)\} aoh_config;", hdr, re.S).group(1)
+    names = re.findall(r"int32_t (\w+);", body)
+    assert names == [n for n, _ in aoh.aoh_config._fields_]
+    assert ctypes.sizeof(aoh.aoh_config) == 4 * len(names)
 
 
 def test_bad_label_rejected(lib):
