@@ -90,9 +90,25 @@ def attended_pairs(T, S, W, streaming):
     return tot
 
 
-def prefill_flops(wl, labels, T):
+def attended_pairs_chunk(T, S, W, K, streaming):
+    """The same under the chunk-eviction rule: a streaming row x of chunk
+    c = x // K sees the sinks and keys c*K - W .. x."""
+    if not streaming:
+        return T * (T + 1) // 2
+    tot = 0
+    for x in range(T):
+        sinks = min(x + 1, S)
+        lo = max(S, (x // K) * K - W, 0)
+        tot += sinks + max(0, x - lo + 1)
+    return tot
+
+
+def prefill_flops(wl, labels, T, chunk=0):
     g = wl.g
-    pairs = sum(attended_pairs(T, wl.sink, wl.window, lab == 1) for lab in labels) * g
+    if chunk:
+        pairs = sum(attended_pairs_chunk(T, wl.sink, wl.window, chunk, lab == 1) for lab in labels) * g
+    else:
+        pairs = sum(attended_pairs(T, wl.sink, wl.window, lab == 1) for lab in labels) * g
     return 4.0 * wl.d_head * pairs
 
 
@@ -323,6 +339,27 @@ def run_native(args):
     chunk_ms = max_over_ranks(cev[0].elapsed_time(cev[1])) / Kp
     ccache.check()
     ccache.close()
+
+    # ---------------- the same chunks under the chunk-eviction rule (chunk = C):
+    # streaming rows see the sinks, the W tokens before their chunk and the chunk
+    ecache = aoh.Cache(1, pwl.n_q_heads, pwl.n_kv_heads, pwl.d_head, T, pwl.sink, pwl.window, plabels, chunk=C)
+    for _ in range(max(W, 3)):
+        ecache.reset()
+        for ch, co in zip(chunks, couts):
+            ecache.prefill(ch[0], ch[1], ch[2], co)
+    ecache.check()
+    barrier()
+    cev[0].record(stream)
+    for _ in range(Kp):
+        ecache.reset()
+        for ch, co in zip(chunks, couts):
+            ecache.prefill(ch[0], ch[1], ch[2], co)
+    cev[1].record(stream)
+    barrier()
+    evict_ms = max_over_ranks(cev[0].elapsed_time(cev[1])) / Kp
+    ecache.check()
+    ecache.close()
+    evict_flops = prefill_flops(pwl, plabels, T, chunk=C)
     del chunks, couts
 
     # ---------------- cpu baseline (oracle on a bounded sample), rank 0 only
@@ -370,6 +407,12 @@ def run_native(args):
         "chunked_prefill": {"chunks": n_chunks, "chunk_tokens": C, "ms": round(chunk_ms, 3),
                             "tflops": round(flops / (chunk_ms * 1e-3) / 1e12, 2),
                             "note": "same 32K prefill as consecutive chunks; each chunk reads the cached prefix"},
+        "chunk_eviction_prefill": {"chunk": C, "ms": round(evict_ms, 3), "flops": evict_flops,
+                                   "tflops": round(evict_flops / (evict_ms * 1e-3) / 1e12, 2),
+                                   "frac": round(evict_flops / (evict_ms * 1e-3) / 1e12 / tf_peak, 4),
+                                   "note": "the same chunks with aoh_config.chunk = C: streaming rows see the sinks, "
+                                           "the W tokens before their chunk and the chunk (attended pairs counted "
+                                           "under that rule)"},
         "e2e": {"value": round(e2e_us, 3), "unit": "us/step", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": K,
         "clocks": clock_info,

@@ -1,0 +1,28 @@
+"""The work counts bench.py divides by: attended (query, key) pairs of a
+prefill, per-token and under the chunk-eviction rule, checked against the
+oracle's masks on small prompts (every allowed pair counted once)."""
+
+import os
+import sys
+
+import numpy as np
+import pytest
+
+from oracle import attention as oatt
+
+sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+import bench  # noqa: E402
+
+
+@pytest.mark.parametrize("T,S,W", [(1, 0, 1), (50, 3, 7), (64, 0, 64), (90, 8, 20), (17, 20, 4)])
+def test_attended_pairs_per_token(T, S, W):
+    for streaming in (False, True):
+        m = oatt.allowed_mask(np.arange(T), np.arange(T), streaming, S, W)
+        assert bench.attended_pairs(T, S, W, streaming) == int(m.sum())
+
+
+@pytest.mark.parametrize("T,S,W,K", [(50, 3, 7, 8), (33, 0, 5, 1), (40, 4, 10, 100), (129, 2, 30, 64)])
+def test_attended_pairs_chunk_rule(T, S, W, K):
+    for streaming in (False, True):
+        m = oatt.allowed_mask(np.arange(T), np.arange(T), streaming, S, W, K)
+        assert bench.attended_pairs_chunk(T, S, W, K, streaming) == int(m.sum())
