@@ -644,6 +644,54 @@ def run_stack(args):
         "peak_note": note}))
 
 
+def run_classify(args):
+    """Effective-rank classification of one Qwen2.5-7B-shaped layer (28 query
+    / 4 KV heads, d_head 128, d_model 3584; seeded N(0,1) bf16 weights whose
+    rows decay geometrically at a random rate per head), timed on the GPU,
+    and the float64 oracle on the same weights on the host cores."""
+    import numpy as np
+    import torch
+
+    from oracle import effective_rank as oer
+    from paper_2608_06849_gb300 import aoh
+    from paper_2608_06849_gb300 import build as aoh_build
+    aoh_build.build()
+    aoh.load()
+    Hq, Hkv, dh, dm, layers = 28, 4, 128, 3584, 28
+    gen = torch.Generator().manual_seed(0)
+    decay = torch.logspace(0, -2, dh, dtype=torch.float64)
+    expo = torch.rand(Hq, 1, 1, generator=gen, dtype=torch.float64) * 1.5
+    wq = (decay[None, :, None] ** expo) * torch.randn(Hq, dh, dm, generator=gen, dtype=torch.float64)
+    wk = decay[None, :, None] ** 0.5 * torch.randn(Hkv, dh, dm, generator=gen, dtype=torch.float64)
+    wq, wk = wq.to(torch.bfloat16), wk.to(torch.bfloat16)
+    dq, dk = wq.cuda(), wk.cuda()
+    for _ in range(max(args.warmup, 3)):
+        aoh.aoh_classify(dq, dk, Hkv, 50)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(3, min(args.steps, 20))
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        labels, er = aoh.aoh_classify(dq, dk, Hkv, 50)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    gram_flops = 2.0 * dh * dh * dm * (Hq + Hkv)
+    t0 = time.perf_counter()
+    want = oer.head_scores(wq.double().numpy(), wk.double().numpy(), Hkv)
+    cpu_s = time.perf_counter() - t0
+    fp64_peak = 1250.0  # GFLOP/s, the nominal FP64 rate of this part
+    print(json.dumps({
+        "workload": f"qwen2.5-7b-classify-layer: Hq={Hq} Hkv={Hkv} d_head={dh} d_model={dm}, sparsity 50%",
+        "ms_per_layer": round(ms, 3), "ms_model_28_layers": round(ms * layers, 2),
+        "labels": labels, "max_rel_err_vs_oracle": float(np.max(np.abs(np.array(er) - want) / want)),
+        "roofline": {"bound": "alu", "achieved": round(gram_flops / (ms * 1e-3) / 1e9, 1), "peak": fp64_peak,
+                     "unit": "GFLOP/s", "frac": round(gram_flops / (ms * 1e-3) / 1e9 / fp64_peak, 4),
+                     "note": "Gram flops (2 d_head^2 d_model per projection) over the whole call; FP64 nominal"},
+        "cpu_baseline": {"value": round(cpu_s * 1e3, 1), "unit": "ms/layer", "cores": os.cpu_count(),
+                         "kind": "oracle", "sample": "the same layer, float64 oracle head_scores"}}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -652,8 +700,9 @@ def main():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--prefill-steps", type=int, default=10)
     ap.add_argument("--prefill-chunks", type=int, default=8)
-    ap.add_argument("--workload", choices=["default", "ragged", "stack"], default="default",
-                    help="default: the headline decode + prefill run; ragged / stack: the other two workloads")
+    ap.add_argument("--workload", choices=["default", "ragged", "stack", "classify"], default="default",
+                    help="default: the headline decode + prefill run; ragged / stack: the other two workloads; "
+                         "classify: the effective-rank head classifier on one layer")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--decode-batch", type=int, default=None, help="smaller decode batch (profiling runs)")
@@ -668,6 +717,8 @@ def main():
         run_ragged(args)
     elif args.workload == "stack":
         run_stack(args)
+    elif args.workload == "classify":
+        run_classify(args)
     else:
         run_native(args)
 

@@ -35,6 +35,7 @@ EXPORTS = [
     "aoh_last_error",
     "aoh_version",
     "aoh_decode_step_noalloc",
+    "aoh_classify",
 ]
 
 
@@ -79,6 +80,7 @@ def load():
         "aoh_last_error": (ctypes.c_char_p, []),
         "aoh_version": (i32, []),
         "aoh_decode_step_noalloc": (i32, [cfgp, u8p, P, i32p, i32, P, P, P, P, P]),
+        "aoh_classify": (i32, [P, P, i32, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), u8p, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -158,6 +160,20 @@ def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_n
         ctypes.byref(cfg), _labels_arr(labels), _ptr(kv_buffer, "kv_buffer", torch.uint8),
         ctypes.cast(ctypes.c_void_p(lens.data_ptr()), ctypes.POINTER(ctypes.c_int32)), int(max_len),
         _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), _ptr(out, "out"), _stream_ptr(stream)))
+
+
+def aoh_classify(w_q, w_k, n_kv_heads, sparsity_pct, stream=None):
+    """Effective-rank labels of one layer. w_q [Hq, d_head, d_model] and
+    w_k [Hkv, d_head, d_model] are contiguous bf16 CUDA tensors. Returns
+    (labels: list of n_kv_heads ints, er: list of n_q_heads floats)."""
+    Hq, dh, dm = w_q.shape
+    if tuple(w_k.shape) != (n_kv_heads, dh, dm):
+        raise ValueError("w_k must be [n_kv_heads, d_head, d_model] like w_q")
+    er = (ctypes.c_double * Hq)()
+    lab = (ctypes.c_uint8 * n_kv_heads)()
+    _check(load().aoh_classify(_ptr(w_q, "w_q"), _ptr(w_k, "w_k"), Hq, n_kv_heads, dh, dm, int(sparsity_pct),
+                               er, lab, _stream_ptr(stream)))
+    return list(lab), list(er)
 
 
 def aoh_cache_lens(cache, batch):
