@@ -227,31 +227,33 @@ aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_la
 
 /*
  * Effective-rank head classification (Sec. 4, Eq. 2-6 and Algorithm 1;
- * Appendix "GQA Extension"), computed on the GPU in fp64. For query head h,
- * M_h = W_K^T W_Q (Eq. 2, the key projection of h's group); its nonzero
- * singular values give ER(h) = exp(entropy of sigma / sum(sigma)) (Eq. 4).
- * A group's score is the mean ER of its query heads; the
+ * Appendix "GQA Extension"), computed on the GPU in fp64, for n_layers
+ * layers at once. For query head h of a layer, M_h = W_K^T W_Q (Eq. 2, the
+ * key projection of h's group); its nonzero singular values give
+ * ER(h) = exp(entropy of sigma / sum(sigma)) (Eq. 4). A group's score is the
+ * mean ER of its query heads; in every layer the
  * ceil((100 - sparsity_pct) * n_kv_heads / 100) lowest groups are labelled
  * retrieval (ties to the lower group index), the rest streaming.
- *   w_q  device bf16 [n_q_heads][d_head][d_model]: W_Q^h is rows
- *        h*d_head .. h*d_head + d_head - 1 of a q_proj weight stored
- *        [n_q_heads * d_head][d_model] (out x in, row-major).
- *   w_k  device bf16 [n_kv_heads][d_head][d_model], the same for k_proj.
- *   d_head 64 or 128; d_model >= 1; sparsity_pct in [0, 100].
- *   er_out     host double [n_q_heads] receiving ER per query head, or NULL.
- *   labels_out host uint8 [n_kv_heads] receiving AOH_RETRIEVAL /
+ *   w_q  device bf16 [n_layers][n_q_heads][d_head][d_model]: per layer,
+ *        W_Q^h is rows h*d_head .. h*d_head + d_head - 1 of a q_proj weight
+ *        stored [n_q_heads * d_head][d_model] (out x in, row-major).
+ *   w_k  device bf16 [n_layers][n_kv_heads][d_head][d_model], likewise.
+ *   d_head 64 or 128; d_model >= 1; sparsity_pct in [0, 100];
+ *   n_layers * (n_q_heads + n_kv_heads) <= 65535.
+ *   er_out     host double [n_layers][n_q_heads] receiving ER, or NULL.
+ *   labels_out host uint8 [n_layers][n_kv_heads] receiving AOH_RETRIEVAL /
  *              AOH_STREAMING, ready for aoh_cache_init.
  * Work: the Gram matrices W W^T (exact bf16 products, fp64 sums), their
  * semi-definite Cholesky factors L, and a one-sided Jacobi SVD of
  * L_K^T L_Q, whose singular values are those of M_h; singular values at or
  * below sigma_max * d_model * eps are dropped as zeros.
- * Allocates temporary device memory stream-ordered (cudaMallocAsync), frees
- * it, and synchronises `stream` before returning. Errors: INVALID,
- * UNSUPPORTED, CUDA.
+ * Allocates temporary device memory stream-ordered (cudaMallocAsync;
+ * about 0.26 MB per matrix at d_head 128), frees it, and synchronises
+ * `stream` before returning. Errors: INVALID, UNSUPPORTED, CUDA.
  */
-aoh_status aoh_classify(const void* w_q, const void* w_k, int32_t n_q_heads, int32_t n_kv_heads,
-                        int32_t d_head, int32_t d_model, int32_t sparsity_pct, double* er_out,
-                        uint8_t* labels_out, void* stream);
+aoh_status aoh_classify(const void* w_q, const void* w_k, int32_t n_layers, int32_t n_q_heads,
+                        int32_t n_kv_heads, int32_t d_head, int32_t d_model, int32_t sparsity_pct,
+                        double* er_out, uint8_t* labels_out, void* stream);
 
 /* Library ABI version (major * 100 + minor); 101 added aoh_config.chunk. */
 int32_t aoh_version(void);

@@ -80,7 +80,7 @@ def load():
         "aoh_last_error": (ctypes.c_char_p, []),
         "aoh_version": (i32, []),
         "aoh_decode_step_noalloc": (i32, [cfgp, u8p, P, i32p, i32, P, P, P, P, P]),
-        "aoh_classify": (i32, [P, P, i32, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), u8p, P]),
+        "aoh_classify": (i32, [P, P, i32, i32, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), u8p, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -163,17 +163,24 @@ def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_n
 
 
 def aoh_classify(w_q, w_k, n_kv_heads, sparsity_pct, stream=None):
-    """Effective-rank labels of one layer. w_q [Hq, d_head, d_model] and
-    w_k [Hkv, d_head, d_model] are contiguous bf16 CUDA tensors. Returns
-    (labels: list of n_kv_heads ints, er: list of n_q_heads floats)."""
-    Hq, dh, dm = w_q.shape
-    if tuple(w_k.shape) != (n_kv_heads, dh, dm):
-        raise ValueError("w_k must be [n_kv_heads, d_head, d_model] like w_q")
-    er = (ctypes.c_double * Hq)()
-    lab = (ctypes.c_uint8 * n_kv_heads)()
-    _check(load().aoh_classify(_ptr(w_q, "w_q"), _ptr(w_k, "w_k"), Hq, n_kv_heads, dh, dm, int(sparsity_pct),
+    """Effective-rank labels. w_q [L, Hq, d_head, d_model] and w_k
+    [L, Hkv, d_head, d_model] (or one layer without the leading L) are
+    contiguous bf16 CUDA tensors. Returns (labels, er): per layer a list of
+    n_kv_heads labels and a list of n_q_heads ER values (one layer: the
+    lists themselves)."""
+    single = w_q.dim() == 3
+    if single:
+        w_q, w_k = w_q.unsqueeze(0), w_k.unsqueeze(0)
+    L, Hq, dh, dm = w_q.shape
+    if tuple(w_k.shape) != (L, n_kv_heads, dh, dm):
+        raise ValueError("w_k must be [layers, n_kv_heads, d_head, d_model] like w_q")
+    er = (ctypes.c_double * (L * Hq))()
+    lab = (ctypes.c_uint8 * (L * n_kv_heads))()
+    _check(load().aoh_classify(_ptr(w_q, "w_q"), _ptr(w_k, "w_k"), L, Hq, n_kv_heads, dh, dm, int(sparsity_pct),
                                er, lab, _stream_ptr(stream)))
-    return list(lab), list(er)
+    labels = [list(lab[l * n_kv_heads:(l + 1) * n_kv_heads]) for l in range(L)]
+    ers = [list(er[l * Hq:(l + 1) * Hq]) for l in range(L)]
+    return (labels[0], ers[0]) if single else (labels, ers)
 
 
 def aoh_cache_lens(cache, batch):

@@ -20,10 +20,16 @@
 //      are disjoint; the singular values are the column norms. Values at or
 //      below sigma_max * d_model * eps are the zeros of a rank-deficient
 //      M_h and are dropped (Eq. 4 sums over nonzero values); ER (Eq. 4) is
-//      exp of the entropy of the normalised singular values.
-//   4. classify_kernel: group score = mean ER of the group's query heads;
-//      the k = ceil((100 - s) * groups / 100) lowest groups (stable order,
-//      ties to the lower index) are retrieval, the rest streaming.
+//      exp of the entropy of the normalised singular values. FP64 is slow
+//      on this part, so a pair costs one fp64 dot product and the column
+//      update: squared norms are carried in shared memory (exact again at
+//      each sweep), and the angle is formed in fp32 (any angle is exact).
+//   4. classify_kernel: per layer, group score = mean ER of the group's
+//      query heads; the k = ceil((100 - s) * groups / 100) lowest groups
+//      (stable order, ties to the lower index) are retrieval, the rest
+//      streaming.
+// One call takes all layers of a model, so every matrix is a CTA of its own
+// and the GPU fills up.
 #include <float.h>
 #include <math.h>
 
@@ -43,13 +49,21 @@ constexpr int kGramThreads = 256;
 constexpr int kMatThreads = 256;
 constexpr int kMaxSweeps = 40;
 
-__global__ void __launch_bounds__(kGramThreads) gram_kernel(const bf16* wq, const bf16* wk, int Hq, int nmat, int dh,
-                                                            int dm, int span, double* part) {
+// Matrices are numbered layer-major: layer l's query projections, then its
+// key projections (nmat = Hq + Hkv per layer).
+__device__ __forceinline__ const bf16* weight_of(const bf16* wq, const bf16* wk, int m, int Hq, int Hkv, int dh,
+                                                 int dm) {
+  const int nmat = Hq + Hkv, l = m / nmat, mi = m % nmat;
+  return mi < Hq ? wq + ((size_t)l * Hq + mi) * dh * dm : wk + ((size_t)l * Hkv + (mi - Hq)) * dh * dm;
+}
+
+__global__ void __launch_bounds__(kGramThreads) gram_kernel(const bf16* wq, const bf16* wk, int Hq, int Hkv, int nall,
+                                                            int dh, int dm, int span, double* part) {
   __shared__ double sa[kGK][kGT + 1], sb[kGK][kGT + 1];
   const int m = blockIdx.z, split = blockIdx.y;
   const int tiles = dh / kGT;
   const int ti = blockIdx.x / tiles, tj = blockIdx.x % tiles;
-  const bf16* W = m < Hq ? wq + (size_t)m * dh * dm : wk + (size_t)(m - Hq) * dh * dm;
+  const bf16* W = weight_of(wq, wk, m, Hq, Hkv, dh, dm);
   const int k0 = split * span, k1 = min(dm, k0 + span);
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   double acc[4][4] = {};
@@ -76,7 +90,7 @@ __global__ void __launch_bounds__(kGramThreads) gram_kernel(const bf16* wq, cons
     }
     __syncthreads();
   }
-  double* out = part + ((size_t)split * nmat + m) * dh * dh;
+  double* out = part + ((size_t)split * nall + m) * dh * dh;
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -106,7 +120,7 @@ __device__ double block_max(double v, double* red) {
 
 // One matrix per CTA: G = sum of the split parts, then G = L L^T in place
 // (lower triangle), written to L with the upper triangle zeroed.
-__global__ void __launch_bounds__(kMatThreads) chol_kernel(const double* part, int nsplit, int nmat, int dh,
+__global__ void __launch_bounds__(kMatThreads) chol_kernel(const double* part, int nsplit, int nall, int dh,
                                                            double* L) {
   extern __shared__ double A[];  // [dh][dh] row-major
   __shared__ double red[32];
@@ -115,7 +129,7 @@ __global__ void __launch_bounds__(kMatThreads) chol_kernel(const double* part, i
   const size_t n2 = (size_t)dh * dh;
   for (int e = threadIdx.x; e < dh * dh; e += kMatThreads) {
     double s = 0.0;
-    for (int p = 0; p < nsplit; ++p) s += part[((size_t)p * nmat + m) * n2 + e];
+    for (int p = 0; p < nsplit; ++p) s += part[((size_t)p * nall + m) * n2 + e];
     A[e] = s;
   }
   __syncthreads();
@@ -163,16 +177,18 @@ __device__ __forceinline__ double warp_sum(double v) {
   return v;
 }
 
-// One query head per CTA: A = L_K^T L_Q, one-sided Jacobi, ER.
+// One query head per CTA (blockIdx.x = layer * Hq + head): A = L_K^T L_Q,
+// one-sided Jacobi, ER.
 __global__ void __launch_bounds__(kMatThreads) er_kernel(const double* L, int Hq, int Hkv, int dh, int dm,
                                                          double* er, int* sweeps_out) {
-  extern __shared__ double A[];  // column-major: column c at A + c * dh
+  extern __shared__ double A[];  // column-major: column c at A + c * dh; then dh squared norms
   __shared__ double red[32];
   __shared__ int rotated;
-  const int h = blockIdx.x, kv = h / (Hq / Hkv);
+  const int hg = blockIdx.x, l = hg / Hq, h = hg % Hq, kv = h / (Hq / Hkv);
   const size_t n2 = (size_t)dh * dh;
-  const double* Lq = L + (size_t)h * n2;
-  const double* Lk = L + (size_t)(Hq + kv) * n2;
+  const double* Lq = L + ((size_t)l * (Hq + Hkv) + h) * n2;
+  const double* Lk = L + ((size_t)l * (Hq + Hkv) + Hq + kv) * n2;
+  double* nrm2 = A + n2;
   for (int e = threadIdx.x; e < dh * dh; e += kMatThreads) {
     const int i = e % dh, j = e / dh;  // A[i][j] = sum_m Lk[m][i] Lq[m][j] over m >= max(i, j)
     double s = 0.0;
@@ -184,10 +200,18 @@ __global__ void __launch_bounds__(kMatThreads) er_kernel(const double* L, int Hq
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   constexpr int kWarps = kMatThreads / 32;
   // a pair counts as orthogonal once |a_p . a_q| <= d_head * eps * |a_p| |a_q|
-  // (the rounding level of a length-d_head dot product)
-  const double rot_tol = dh * DBL_EPSILON;
+  // (the rounding level of a length-d_head dot product), tested squared
+  const double rot_tol2 = (dh * DBL_EPSILON) * (dh * DBL_EPSILON);
   int sweep = 0;
   for (; sweep < kMaxSweeps; ++sweep) {
+    // squared column norms, exact at the start of each sweep and carried
+    // through its rotations
+    for (int c = threadIdx.x; c < dh; c += kMatThreads) {
+      const double* a = A + (size_t)c * dh;
+      double s2 = 0.0;
+      for (int i = 0; i < dh; ++i) s2 = fma(a[i], a[i], s2);
+      nrm2[c] = s2;
+    }
     if (threadIdx.x == 0) rotated = 0;
     __syncthreads();
     for (int r = 0; r < dh - 1; ++r) {
@@ -196,27 +220,30 @@ __global__ void __launch_bounds__(kMatThreads) er_kernel(const double* L, int Hq
         rr_pair(dh, r, k, p, q);
         double* ap = A + (size_t)p * dh;
         double* aq = A + (size_t)q * dh;
-        double al = 0.0, be = 0.0, ga = 0.0;
-        for (int i = lane; i < dh; i += 32) {
-          const double x = ap[i], y = aq[i];
-          al = fma(x, x, al);
-          be = fma(y, y, be);
-          ga = fma(x, y, ga);
-        }
-        al = warp_sum(al);
-        be = warp_sum(be);
+        const double al = nrm2[p], be = nrm2[q];
+        double ga = 0.0;
+        for (int i = lane; i < dh; i += 32) ga = fma(ap[i], aq[i], ga);
         ga = warp_sum(ga);
-        if (fabs(ga) > rot_tol * sqrt(al * be) && ga != 0.0) {
-          const double zeta = (be - al) / (2.0 * ga);
-          const double t = fabs(zeta) > 1e150 ? 0.5 / zeta
-                                               : copysign(1.0, zeta) / (fabs(zeta) + sqrt(1.0 + zeta * zeta));
-          const double c = 1.0 / sqrt(1.0 + t * t), s = c * t;
+        if (ga != 0.0 && ga * ga > rot_tol2 * al * be) {
+          // The angle only steers convergence: any (c, s) with c^2 + s^2 = 1
+          // to fp64 precision is an exact orthogonal transform, so tan is
+          // formed in fp32 and c, s from it in fp64.
+          const float zeta = (float)(be - al) / (2.0f * (float)ga);
+          const float tf = fabsf(zeta) > 1e18f ? 0.5f / zeta
+                                               : copysignf(1.0f, zeta) / (fabsf(zeta) + sqrtf(1.0f + zeta * zeta));
+          const double t = tf;
+          const double c = rsqrt(1.0 + t * t), s = c * t;
           for (int i = lane; i < dh; i += 32) {
             const double x = ap[i], y = aq[i];
-            ap[i] = c * x - s * y;
-            aq[i] = s * x + c * y;
+            ap[i] = fma(c, x, -s * y);
+            aq[i] = fma(s, x, c * y);
           }
-          if (lane == 0) rotated = 1;
+          if (lane == 0) {
+            const double cc = c * c, ss = s * s, cs2 = 2.0 * c * s * ga;
+            nrm2[p] = fmax(fma(cc, al, fma(ss, be, -cs2)), 0.0);
+            nrm2[q] = fmax(fma(ss, al, fma(cc, be, cs2)), 0.0);
+            rotated = 1;
+          }
         }
       }
       __syncthreads();
@@ -244,13 +271,16 @@ __global__ void __launch_bounds__(kMatThreads) er_kernel(const double* L, int Hq
   }
   ent = block_sum(ent, red);
   if (threadIdx.x == 0) {
-    er[h] = exp(ent);
-    sweeps_out[h] = sweep;
+    er[hg] = exp(ent);
+    sweeps_out[hg] = sweep;
   }
 }
 
-__global__ void classify_kernel(const double* er, int Hq, int Hkv, int sparsity_pct, uint8_t* labels) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+// One layer per block (blockIdx.x), one thread.
+__global__ void classify_kernel(const double* er_all, int Hq, int Hkv, int sparsity_pct, uint8_t* labels_all) {
+  if (threadIdx.x != 0) return;
+  const double* er = er_all + (size_t)blockIdx.x * Hq;
+  uint8_t* labels = labels_all + (size_t)blockIdx.x * Hkv;
   const int g = Hq / Hkv;
   double score[kMaxKvHeads];
   int order[kMaxKvHeads];
@@ -278,15 +308,16 @@ __global__ void classify_kernel(const double* er, int Hq, int Hkv, int sparsity_
 
 using namespace aoh;
 
-extern "C" aoh_status aoh_classify(const void* w_q, const void* w_k, int32_t n_q_heads, int32_t n_kv_heads,
-                                   int32_t d_head, int32_t d_model, int32_t sparsity_pct, double* er_out,
-                                   uint8_t* labels_out, void* stream) {
+extern "C" aoh_status aoh_classify(const void* w_q, const void* w_k, int32_t n_layers, int32_t n_q_heads,
+                                   int32_t n_kv_heads, int32_t d_head, int32_t d_model, int32_t sparsity_pct,
+                                   double* er_out, uint8_t* labels_out, void* stream) {
   auto fail = [](aoh_status st, const char* msg) {
     record_error(msg);
     return st;
   };
   if (!w_q || !w_k || !labels_out)
     return fail(AOH_ERR_INVALID, "aoh_classify: w_q, w_k and labels_out must not be NULL");
+  if (n_layers < 1 || n_layers > 65535) return fail(AOH_ERR_INVALID, "aoh_classify: n_layers outside [1, 65535]");
   if (n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads)
     return fail(AOH_ERR_INVALID, "aoh_classify: n_q_heads must be a positive multiple of n_kv_heads");
   if (n_kv_heads > kMaxKvHeads) return fail(AOH_ERR_UNSUPPORTED, "aoh_classify: more than 64 KV heads");
@@ -296,48 +327,52 @@ extern "C" aoh_status aoh_classify(const void* w_q, const void* w_k, int32_t n_q
     return fail(AOH_ERR_INVALID, "aoh_classify: sparsity_pct outside [0, 100]");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int dh = d_head, nmat = n_q_heads + n_kv_heads, tiles = dh / kGT;
+  const int nall = n_layers * nmat, nq = n_layers * n_q_heads;
+  if ((long long)n_layers * nmat > 65535) return fail(AOH_ERR_INVALID, "aoh_classify: too many matrices in one call");
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return fail(AOH_ERR_CUDA, "aoh_classify: device query failed");
   // split d_model so that the Gram grid covers about two waves, >= 256 columns a split
-  int nsplit = (2 * sms + nmat * tiles * tiles - 1) / (nmat * tiles * tiles);
+  int nsplit = (2 * sms + nall * tiles * tiles - 1) / (nall * tiles * tiles);
   nsplit = std::max(1, std::min(nsplit, std::max(1, d_model / 256)));
   nsplit = std::min(nsplit, 16);
   const int span = ((d_model + nsplit - 1) / nsplit + kGK - 1) / kGK * kGK;
   nsplit = (d_model + span - 1) / span;
   const size_t n2 = (size_t)dh * dh;
-  const size_t bytes = ((size_t)nsplit * nmat * n2 + (size_t)nmat * n2 + n_q_heads) * sizeof(double) +
-                       n_q_heads * sizeof(int) + 64;
+  const size_t bytes = ((size_t)nsplit * nall * n2 + (size_t)nall * n2 + nq) * sizeof(double) + nq * sizeof(int) +
+                       (size_t)n_layers * n_kv_heads + 64;
   void* scratch = nullptr;
   e = cudaMallocAsync(&scratch, bytes, s);
   if (e != cudaSuccess) return fail(AOH_ERR_CUDA, "aoh_classify: cudaMallocAsync failed");
   double* part = static_cast<double*>(scratch);
-  double* L = part + (size_t)nsplit * nmat * n2;
-  double* er = L + (size_t)nmat * n2;
-  int* sweeps = reinterpret_cast<int*>(er + n_q_heads);
-  uint8_t* labels = reinterpret_cast<uint8_t*>(sweeps + n_q_heads);
+  double* L = part + (size_t)nsplit * nall * n2;
+  double* er = L + (size_t)nall * n2;
+  int* sweeps = reinterpret_cast<int*>(er + nq);
+  uint8_t* labels = reinterpret_cast<uint8_t*>(sweeps + nq);
   const int smem = (int)(n2 * sizeof(double));
+  const int smem_er = (int)((n2 + dh) * sizeof(double));
   static bool attr_set = false;
   if (!attr_set) {
     e = cudaFuncSetAttribute(chol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 128 * 128 * 8);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(er_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 128 * 128 * 8);
+      e = cudaFuncSetAttribute(er_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (128 * 128 + 128) * 8);
     if (e != cudaSuccess) {
       cudaFreeAsync(scratch, s);
       return fail(AOH_ERR_CUDA, "aoh_classify: cudaFuncSetAttribute failed");
     }
     attr_set = true;
   }
-  gram_kernel<<<dim3(tiles * tiles, nsplit, nmat), kGramThreads, 0, s>>>(
-      static_cast<const bf16*>(w_q), static_cast<const bf16*>(w_k), n_q_heads, nmat, dh, d_model, span, part);
-  chol_kernel<<<nmat, kMatThreads, smem, s>>>(part, nsplit, nmat, dh, L);
-  er_kernel<<<n_q_heads, kMatThreads, smem, s>>>(L, n_q_heads, n_kv_heads, dh, d_model, er, sweeps);
-  classify_kernel<<<1, 32, 0, s>>>(er, n_q_heads, n_kv_heads, sparsity_pct, labels);
+  gram_kernel<<<dim3(tiles * tiles, nsplit, nall), kGramThreads, 0, s>>>(static_cast<const bf16*>(w_q),
+                                                                          static_cast<const bf16*>(w_k), n_q_heads,
+                                                                          n_kv_heads, nall, dh, d_model, span, part);
+  chol_kernel<<<nall, kMatThreads, smem, s>>>(part, nsplit, nall, dh, L);
+  er_kernel<<<nq, kMatThreads, smem_er, s>>>(L, n_q_heads, n_kv_heads, dh, d_model, er, sweeps);
+  classify_kernel<<<n_layers, 32, 0, s>>>(er, n_q_heads, n_kv_heads, sparsity_pct, labels);
   e = cudaGetLastError();
-  if (e == cudaSuccess) e = cudaMemcpyAsync(labels_out, labels, n_kv_heads, cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess && er_out)
-    e = cudaMemcpyAsync(er_out, er, n_q_heads * sizeof(double), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(labels_out, labels, (size_t)n_layers * n_kv_heads, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess && er_out) e = cudaMemcpyAsync(er_out, er, nq * sizeof(double), cudaMemcpyDeviceToHost, s);
   const cudaError_t f = cudaFreeAsync(scratch, s);
   if (e == cudaSuccess) e = f;
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);

@@ -114,12 +114,14 @@ def test_classify_rejects_bad_arguments_on_host(lib):
     """Argument errors are reported before any CUDA call (no GPU needed)."""
     lab = (ctypes.c_uint8 * 2)()
     fake = ctypes.c_void_p(1 << 20)  # never dereferenced
-    assert lib.aoh_classify(None, fake, 8, 2, 128, 512, 50, None, lab, None) == 1
-    assert lib.aoh_classify(fake, fake, 8, 3, 128, 512, 50, None, lab, None) == 1
-    assert lib.aoh_classify(fake, fake, 8, 2, 96, 512, 50, None, lab, None) == 5
-    assert lib.aoh_classify(fake, fake, 8, 2, 128, 0, 50, None, lab, None) == 1
-    assert lib.aoh_classify(fake, fake, 8, 2, 128, 512, 101, None, lab, None) == 1
-    assert lib.aoh_classify(fake, fake, 8, 2, 128, 512, 50, None, None, None) == 1
+    assert lib.aoh_classify(None, fake, 1, 8, 2, 128, 512, 50, None, lab, None) == 1
+    assert lib.aoh_classify(fake, fake, 0, 8, 2, 128, 512, 50, None, lab, None) == 1
+    assert lib.aoh_classify(fake, fake, 1, 8, 3, 128, 512, 50, None, lab, None) == 1
+    assert lib.aoh_classify(fake, fake, 1, 8, 2, 96, 512, 50, None, lab, None) == 5
+    assert lib.aoh_classify(fake, fake, 1, 8, 2, 128, 0, 50, None, lab, None) == 1
+    assert lib.aoh_classify(fake, fake, 1, 8, 2, 128, 512, 101, None, lab, None) == 1
+    assert lib.aoh_classify(fake, fake, 1, 8, 2, 128, 512, 50, None, None, None) == 1
+    assert lib.aoh_classify(fake, fake, 5000, 8, 8, 128, 512, 50, None, lab, None) == 1  # > 65535 matrices
 
 
 def test_bad_label_rejected(lib):

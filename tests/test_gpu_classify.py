@@ -139,3 +139,22 @@ def test_budget_edges_and_ties():
         assert er[kv * g] == er[0] and er[kv * g + 1] == er[1]
     lab75, er75 = _classify(wq, wk, 75)
     assert lab75.tolist() == oer.classify_groups(er75, Hkv, 75).tolist() == [0, 1, 1, 1]
+
+
+def test_layers_in_one_call():
+    """Several layers in one call give each layer's own result (labels by
+    layer, ER within 1e-12 of the one-layer calls, whose d_model split, and
+    so summation order, may differ) and agree with the oracle."""
+    ensure_lib()
+    rng = np.random.default_rng(13)
+    L, Hq, Hkv, dh, dm = 3, 8, 2, 128, 256
+    wq = _bf16(rng.standard_normal((L, Hq, dh, dm)) * rng.uniform(0.2, 2.0, size=(L, Hq, dh, 1)))
+    wk = _bf16(rng.standard_normal((L, Hkv, dh, dm)))
+    labels, ers = aoh.aoh_classify(_dev(wq), _dev(wk), Hkv, 50)
+    assert len(labels) == L and len(ers) == L
+    for l in range(L):
+        lab1, er1 = _classify(wq[l], wk[l], 50)
+        np.testing.assert_allclose(ers[l], er1, rtol=1e-12)
+        want = oer.head_scores(wq[l], wk[l], Hkv)
+        np.testing.assert_allclose(ers[l], want, rtol=1e-9)
+        _check_labels(np.array(labels[l]), np.array(ers[l]), want, Hkv, 50)
