@@ -21,10 +21,14 @@ Modules
                the d_head proxy C_h of Eq. 5-6, a QR route), and the
                group-level classification of Algorithm 1 plus the GQA
                extension appendix.
+  h2share      index-only cross-layer sparse attention (the H2Share
+               section): anchor-group importance and top-k selection,
+               sparse attention at borrowed positions, the Eq. sim head
+               similarity and the group mapping.
 
 Parity status: every function here is pinned by ``tests/test_oracle_*.py``
 against closed forms, brute force, a textbook library routine or values the
 paper prints. None is "parity unpinned".
 """
 
-from . import attention, effective_rank, kv_memory  # noqa: F401
+from . import attention, effective_rank, h2share, kv_memory  # noqa: F401

@@ -80,6 +80,20 @@ KV_MUTANTS = {
 }
 
 
+H2_MUTANTS = {
+    "similarity_transposed_key_product": ("num = np.trace((Wq_a @ Wq_r.T) @ (Wk_r @ Wk_a.T))",
+                                          "num = np.trace((Wq_a @ Wq_r.T) @ (Wk_a @ Wk_r.T))"),
+    "similarity_no_norm": ("return num / np.sqrt(na * nr)", "return num / np.sqrt(na)"),
+    "importance_unnormalised": ("p = p / p.sum(axis=1, keepdims=True)\n    return p.sum(axis=0)",
+                                "return p.sum(axis=0)"),
+    "topk_ties_high": ("key=lambda j: (-imp[j], j)", "key=lambda j: (-imp[j], -j)"),
+    "sparse_no_scale": ("s = (q @ k.T) / np.sqrt(q.shape[1])\n    s = s - s.max(axis=1, keepdims=True)\n    p = np.exp(s)\n    p = p / p.sum(axis=1, keepdims=True)\n    return p @ v",
+                        "s = (q @ k.T)\n    s = s - s.max(axis=1, keepdims=True)\n    p = np.exp(s)\n    p = p / p.sum(axis=1, keepdims=True)\n    return p @ v"),
+    "mapping_ties_high": ("if sim[a, r] > sim[best, r]:", "if sim[a, r] >= sim[best, r]:"),
+    "group_mean_max": ("out[ga, gr] = np.mean(vals)", "out[ga, gr] = np.max(vals)"),
+}
+
+
 def _mutated(modname, old, new):
     path = os.path.join(os.path.dirname(SRC), modname + ".py")
     src = open(path).read()
@@ -93,7 +107,7 @@ def _mutated(modname, old, new):
 def _failures(test_module_name, monkeypatch, modname, mod):
     monkeypatch.setattr(oracle, modname, mod)
     tm = importlib.import_module(test_module_name)
-    monkeypatch.setattr(tm, {"effective_rank": "er", "kv_memory": "kvm"}[modname], mod)
+    monkeypatch.setattr(tm, {"effective_rank": "er", "kv_memory": "kvm", "h2share": "hs"}[modname], mod)
     failed = 0
     for name in dir(tm):
         if not name.startswith("test_"):
@@ -124,3 +138,9 @@ def test_er_pins_catch_mutant(name, monkeypatch):
 def test_kv_pins_catch_mutant(name, monkeypatch):
     mod = _mutated("kv_memory", *KV_MUTANTS[name])
     assert _failures("test_oracle_kv_memory", monkeypatch, "kv_memory", mod) > 0
+
+
+@pytest.mark.parametrize("name", sorted(H2_MUTANTS))
+def test_h2share_pins_catch_mutant(name, monkeypatch):
+    mod = _mutated("h2share", *H2_MUTANTS[name])
+    assert _failures("test_oracle_h2share", monkeypatch, "h2share", mod) > 0
