@@ -77,6 +77,23 @@ def decode_bytes(lens_before, labels, wl):
     return total
 
 
+def reuse_bytes(lens_before, labels, wl, top_k):
+    """Algorithmic HBM bytes of one H2Share reuse step: min(top_k, t + 1)
+    borrowed K/V rows per retrieval head, the ring rows of streaming heads,
+    the new token's K/V read and appended, the index lists, q and out."""
+    D = wl.d_head
+    row = D * 2
+    total = 0
+    for t in lens_before:
+        for lab in labels:
+            rows = min(top_k, t + 1) if lab == 0 else min(t + 1, wl.sink + wl.window)
+            total += (rows - 1) * row * 2 + row * 2 * 2
+            if lab == 0:
+                total += min(top_k, t + 1) * 4
+        total += wl.n_q_heads * D * 2 * 2
+    return total
+
+
 def attended_pairs(T, S, W, streaming):
     """Number of (query, key) pairs a head attends in a causal prefill of T tokens."""
     if not streaming:
@@ -232,7 +249,8 @@ def run_native(args):
     # ---------------- decode leg (headline)
     wl, labels = decode_workload(args.decode_batch, args.decode_ctx)
     B, D, T0 = wl.batch, wl.d_head, wl.prefill_len
-    total_steps = W + K + K + 2   # warmup, timed, e2e
+    KH = min(K, 16)                                   # H2Share leg steps
+    total_steps = W + K + K + 2 + 2 * (W + KH)         # warmup, timed, e2e, anchor, reuse
     cache = aoh.Cache(B, wl.n_q_heads, wl.n_kv_heads, D, T0 + total_steps + 8, wl.sink, wl.window, labels)
     kfill = randn_bf16((B, T0, wl.n_kv_heads, D), replica_seed(7001, rank), "cuda")
     vfill = randn_bf16((B, T0, wl.n_kv_heads, D), replica_seed(7002, rank), "cuda")
@@ -283,6 +301,42 @@ def run_native(args):
     e1.record(stream)
     barrier()
     e2e_us = max_over_ranks(e0.elapsed_time(e1)) * 1000.0 / K
+
+    # ---------------- H2Share leg on the same cache: anchor steps (decode +
+    # scores + top-k selection), then reuse steps over the borrowed positions
+    top_k = args.h2_top_k
+    retr = [h for h in range(wl.n_kv_heads) if labels[h] == 0]
+    idx = torch.empty((B, len(retr), top_k), dtype=torch.int32, device="cuda")
+    gmap = list(range(len(retr)))
+    for s_ in range(W):
+        cache.decode_step_anchor(*inputs[s_], out, top_k, idx)
+    barrier()
+    e0.record(stream)
+    for s_ in range(KH):
+        cache.decode_step_anchor(*inputs[W + s_], out, top_k, idx)
+    e1.record(stream)
+    barrier()
+    anchor_us = max_over_ranks(e0.elapsed_time(e1)) * 1000.0 / KH
+    for s_ in range(W):
+        cache.decode_step_reuse(*inputs[s_], out, idx, top_k, gmap)
+    cache.check()
+    lens_r = cache.lens()
+    barrier()
+    e0.record(stream)
+    for s_ in range(KH):
+        cache.decode_step_reuse(*inputs[W + s_], out, idx, top_k, gmap)
+    e1.record(stream)
+    barrier()
+    reuse_us = max_over_ranks(e0.elapsed_time(e1)) * 1000.0 / KH
+    cache.check()
+    r_bytes = sum(reuse_bytes([x + s_ for x in lens_r], labels, wl, top_k) for s_ in range(KH)) / KH
+    h2 = {"top_k": top_k, "anchor_us_per_step": round(anchor_us, 2),
+          "anchor_over_decode": round(anchor_us / dec_us_step, 4),
+          "reuse_us_per_step": round(reuse_us, 2), "reuse_bytes_per_step": int(r_bytes),
+          "reuse_hbm_gbs": round(r_bytes / (reuse_us * 1e-6) / 1e9, 1),
+          "reuse_speedup_vs_decode": round(dec_us_step / reuse_us, 2),
+          "note": "same cache and inputs as the decode leg; the reuse layer borrows the anchor's positions "
+                  "(identity group map); top_k is a reading (the paper gives none)"}
     cache.close()
     del cache, inputs
     torch.cuda.empty_cache()
@@ -413,6 +467,7 @@ def run_native(args):
                                    "note": "the same chunks with aoh_config.chunk = C: streaming rows see the sinks, "
                                            "the W tokens before their chunk and the chunk (attended pairs counted "
                                            "under that rule)"},
+        "h2share": h2,
         "e2e": {"value": round(e2e_us, 3), "unit": "us/step", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": K,
         "clocks": clock_info,
@@ -716,6 +771,7 @@ def main():
                     help="default: the headline decode + prefill run; ragged / stack: the other two workloads; "
                          "classify: the effective-rank head classifier on one layer")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--h2-top-k", type=int, default=2048, help="positions an H2Share anchor step selects")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--decode-batch", type=int, default=None, help="smaller decode batch (profiling runs)")
     ap.add_argument("--decode-ctx", type=int, default=None, help="smaller decode context (profiling runs)")

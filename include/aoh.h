@@ -152,6 +152,49 @@ aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T,
 aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,
                            void* out, void* stream);
 
+/*
+ * H2Share anchor layer (the paper's H2Share section; GQA extension
+ * appendix): an ordinary decode step (as aoh_decode_step) that also selects,
+ * for every sequence b and retrieval KV head, the positions a reuse layer of
+ * the same block will borrow. The importance of position j is the sum over
+ * the group's query heads of their attention probabilities at j (positions
+ * 0..t, the new token included); the min(top_k, t + 1) most important
+ * positions are kept, ties to the lower position, in increasing order.
+ *   top_k    >= 1.
+ *   indices  device int32 [B][n_r][top_k] (n_r = retrieval KV heads, in
+ *            increasing KV-head index), written on the stream; entries past
+ *            min(top_k, t + 1) are -1.
+ * Needs d_head 128 (the tensor-core decode). The first call allocates a
+ * workspace of about B * n_r * max_seq * (group size + 1) floats in the handle
+ * (a cudaMalloc, which synchronises the device); aoh_cache_destroy frees it.
+ * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
+ */
+aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,
+                                  void* out, int32_t top_k, int32_t* indices, void* stream);
+
+/*
+ * H2Share reuse layer: a decode step whose retrieval heads attend only to
+ * their own K/V at positions borrowed from the block's anchor layer (no K/V
+ * crosses layers); streaming heads decode as usual, and the new token is
+ * appended for every head as in aoh_decode_step.
+ *   indices          device int32 [B][n_anchor_groups][top_k] from
+ *                    aoh_decode_step_anchor at the same step (the anchor
+ *                    layer holds the same sequence lengths).
+ *   n_anchor_groups  the anchor layer's retrieval KV heads, 1..64.
+ *   top_k            as given to the anchor step.
+ *   group_map        host int32 [n_r]: for this layer's i-th retrieval KV
+ *                    head, the anchor retrieval head (0..n_anchor_groups-1)
+ *                    whose positions it borrows (the paper maps each reuse
+ *                    group to its most similar anchor group, Eq. sim).
+ * Retrieval head i of sequence b attends to the first min(top_k, t + 1)
+ * entries of its list; entries outside [0, t] are clamped into it (the
+ * reads stay in bounds, the result is then unspecified).
+ * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
+ */
+aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,
+                                 void* out, const int32_t* indices, int32_t n_anchor_groups, int32_t top_k,
+                                 const int32_t* group_map, void* stream);
+
 /* Copy the host-side lengths (tokens held per sequence) into lens_out [B]. */
 aoh_status aoh_cache_lens(const aoh_cache* cache, int32_t* lens_out);
 

@@ -36,6 +36,8 @@ EXPORTS = [
     "aoh_version",
     "aoh_decode_step_noalloc",
     "aoh_classify",
+    "aoh_decode_step_anchor",
+    "aoh_decode_step_reuse",
 ]
 
 
@@ -72,6 +74,8 @@ def load():
         "aoh_cache_init": (i32, [cfgp, u8p, P, ctypes.c_size_t, ctypes.POINTER(P)]),
         "aoh_prefill": (i32, [P, P, P, i32, i32p, P, P, P]),
         "aoh_decode_step": (i32, [P, P, P, P, P, P]),
+        "aoh_decode_step_anchor": (i32, [P, P, P, P, P, i32, P, P]),
+        "aoh_decode_step_reuse": (i32, [P, P, P, P, P, P, i32, i32, i32p, P]),
         "aoh_cache_lens": (i32, [P, i32p]),
         "aoh_cache_region": (i32, [P, i32, i32, szp, szp, i32p]),
         "aoh_cache_reset": (i32, [P, P]),
@@ -151,6 +155,23 @@ def aoh_decode_step(q, k_new, v_new, cache, out, stream=None):
                                   _ptr(out, "out"), _stream_ptr(stream)))
 
 
+def aoh_decode_step_anchor(q, k_new, v_new, cache, out, top_k, indices, stream=None):
+    """H2Share anchor step; indices: contiguous int32 CUDA tensor [B, n_r, top_k]."""
+    _check(load().aoh_decode_step_anchor(_ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), cache,
+                                         _ptr(out, "out"), int(top_k), _ptr(indices, "indices", torch.int32),
+                                         _stream_ptr(stream)))
+
+
+def aoh_decode_step_reuse(q, k_new, v_new, cache, out, indices, top_k, group_map, stream=None):
+    """H2Share reuse step; indices [B, n_anchor_groups, top_k] int32 CUDA tensor
+    from the anchor step; group_map: host list, one anchor group per
+    retrieval KV head of this layer."""
+    gm = (ctypes.c_int32 * max(1, len(group_map)))(*[int(x) for x in group_map])
+    _check(load().aoh_decode_step_reuse(_ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), cache,
+                                        _ptr(out, "out"), _ptr(indices, "indices", torch.int32),
+                                        int(indices.shape[1]), int(top_k), gm, _stream_ptr(stream)))
+
+
 def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream=None):
     """The allocation-free decode step: ``kv_buffer`` (CUDA uint8) and ``lens``
     (CUDA int32 [B], advanced by one on the device) belong to the caller."""
@@ -227,6 +248,12 @@ class Cache:
 
     def decode_step(self, q, k_new, v_new, out, stream=None):
         aoh_decode_step(q, k_new, v_new, self.handle, out, stream)
+
+    def decode_step_anchor(self, q, k_new, v_new, out, top_k, indices, stream=None):
+        aoh_decode_step_anchor(q, k_new, v_new, self.handle, out, top_k, indices, stream)
+
+    def decode_step_reuse(self, q, k_new, v_new, out, indices, top_k, group_map, stream=None):
+        aoh_decode_step_reuse(q, k_new, v_new, self.handle, out, indices, top_k, group_map, stream)
 
     def lens(self):
         return aoh_cache_lens(self.handle, self.batch)

@@ -125,6 +125,8 @@ struct aoh_cache {
   // prefill work list (device), grown on demand
   int4* d_work = nullptr;
   size_t work_cap = 0;
+  // H2Share anchor workspace (scores, importance), allocated on first use
+  float* d_h2 = nullptr;
 };
 
 extern "C" {
@@ -226,6 +228,7 @@ void aoh_cache_destroy(aoh_cache* cache) {
   if (!cache) return;
   if (cache->meta) cudaFree(cache->meta);
   if (cache->d_work) cudaFree(cache->d_work);
+  if (cache->d_h2) cudaFree(cache->d_h2);
   delete cache;
 }
 
@@ -353,21 +356,26 @@ aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, c
   return AOH_OK;
 }
 
-aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, aoh_cache* cache, void* out,
-                           void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Host checks shared by the decode entry points; fills `a` for the step and
+// the step's total rows (every retrieval row; ring rows of streaming heads).
+aoh_status prepare_decode(const void* q, const void* k_new, const void* v_new, aoh_cache* cache, void* out,
+                          DecodeArgs& a, long long& total) {
   if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
   if (!q || !k_new || !v_new || !out) return fail(AOH_ERR_INVALID, "q, k_new, v_new and out must not be NULL");
   if (!aligned(q, 16) || !aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(out, 16))
     return fail(AOH_ERR_INVALID, "q, k_new, v_new and out must be 16-byte aligned");
   const CacheGeom& g = cache->geom;
-  long long total = 0;
+  total = 0;
   for (int b = 0; b < g.B; ++b) {
     if (g.n_r > 0 && cache->lens[b] + 1 > g.max_seq)
       return fail(AOH_ERR_CAPACITY, "sequence %d holds %d tokens; max_seq is %d", b, cache->lens[b], g.max_seq);
     const long long t1 = cache->lens[b] + 1;
     total += g.n_r * t1 + g.n_s * std::min<long long>(t1, g.S + g.W);
   }
-  DecodeArgs a;
   a.tcr = cache->tcr;
   a.tcs = cache->tcs;
   a.geom = g;
@@ -382,10 +390,96 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
   a.gcounters = cache->d_gcounters;
   a.done = cache->d_done;
   a.err = cache->d_err;
-  a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
+  return AOH_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, aoh_cache* cache, void* out,
+                           void* stream) {
+  DecodeArgs a;
+  long long total = 0;
+  const aoh_status st = prepare_decode(q, k_new, v_new, cache, out, a, total);
+  if (st != AOH_OK) return st;
+  const CacheGeom& g = cache->geom;
+  a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
   cudaError_t e = launch_decode(a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");
+  for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
+  return AOH_OK;
+}
+
+aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* v_new, aoh_cache* cache, void* out,
+                                  int32_t top_k, int32_t* indices, void* stream) {
+  DecodeArgs a;
+  long long total = 0;
+  const aoh_status st = prepare_decode(q, k_new, v_new, cache, out, a, total);
+  if (st != AOH_OK) return st;
+  const CacheGeom& g = cache->geom;
+  if (top_k < 1) return fail(AOH_ERR_INVALID, "top_k must be >= 1");
+  if (g.n_r > 0 && !indices) return fail(AOH_ERR_INVALID, "indices must not be NULL");
+  if (!decode_uses_tc(g.D, g.G))
+    return fail(AOH_ERR_UNSUPPORTED, "the anchor step needs the d_head 128 tensor-core decode");
+  if (g.n_r > 0 && !cache->d_h2) {
+    // scores [B][n_r][G][max_seq], importance, chunk states, histograms
+    const size_t n = h2_workspace_floats(g.B, g.n_r, g.G, g.max_seq);
+    cudaError_t e = cudaMalloc(&cache->d_h2, n * sizeof(float));
+    if (e == cudaSuccess) e = h2_workspace_clear(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, (cudaStream_t)stream);
+    if (e != cudaSuccess) {
+      if (cache->d_h2) cudaFree(cache->d_h2);
+      cache->d_h2 = nullptr;
+      return cuda_fail(e, "anchor workspace allocation");
+    }
+  }
+  if (g.n_r > 0) h2_decode_outputs(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, &a.scores, &a.score_stats);
+  a.score_stride = g.max_seq;
+  a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = launch_decode(a, s);
+  if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");
+  for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
+  if (g.n_r > 0) {
+    e = launch_h2_topk(cache->d_h2, g.max_seq, cache->d_lens, g.B, g.n_r, g.G, top_k, indices, s);
+    if (e != cudaSuccess) return cuda_fail(e, "top-k kernel launch");
+  }
+  return AOH_OK;
+}
+
+aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v_new, aoh_cache* cache, void* out,
+                                 const int32_t* indices, int32_t n_anchor_groups, int32_t top_k,
+                                 const int32_t* group_map, void* stream) {
+  DecodeArgs a;
+  long long total = 0;
+  const aoh_status st = prepare_decode(q, k_new, v_new, cache, out, a, total);
+  if (st != AOH_OK) return st;
+  const CacheGeom& g = cache->geom;
+  if (!decode_cc_supported(g.D, g.G)) return fail(AOH_ERR_UNSUPPORTED, "group size not compiled for the reuse step");
+  if (top_k < 1) return fail(AOH_ERR_INVALID, "top_k must be >= 1");
+  if (g.n_r > 0) {
+    if (!indices || !group_map) return fail(AOH_ERR_INVALID, "indices and group_map must not be NULL");
+    if (!aligned(indices, 4)) return fail(AOH_ERR_INVALID, "indices must be 4-byte aligned");
+    if (n_anchor_groups < 1 || n_anchor_groups > kMaxKvHeads)
+      return fail(AOH_ERR_INVALID, "n_anchor_groups must be in [1, %d]", kMaxKvHeads);
+    for (int i = 0; i < g.n_r; ++i)
+      if (group_map[i] < 0 || group_map[i] >= n_anchor_groups)
+        return fail(AOH_ERR_INVALID, "group_map[%d] = %d is outside [0, %d)", i, group_map[i], n_anchor_groups);
+    for (int i = 0; i < g.n_r; ++i) a.idx_map[i] = (uint8_t)group_map[i];
+  }
+  // every retrieval item now holds min(top_k, t + 1) rows
+  total = 0;
+  for (int b = 0; b < g.B; ++b) {
+    const long long t1 = cache->lens[b] + 1;
+    total += g.n_r * std::min<long long>(t1, top_k) + g.n_s * std::min<long long>(t1, g.S + g.W);
+  }
+  a.idx = g.n_r > 0 ? indices : nullptr;
+  a.top_k = top_k;
+  a.n_idx_groups = n_anchor_groups;
+  a.n_ctas = decode_cc_ctas(total, cache->num_sms);
+  cudaError_t e = launch_decode_cc(a, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "reuse decode kernel launch");
   for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
   return AOH_OK;
 }

@@ -1,8 +1,9 @@
 // Split-KV flash-decode for head-heterogeneous attention on CUDA cores (Sec.
 // 5, "Decode Stage", Eq. 8): one new token per sequence; retrieval KV heads
 // attend over their whole history, streaming KV heads over their S sink + W
-// window slots. This kernel serves d_head 64; d_head 128 runs on the tensor
-// cores (decode_tc.cu).
+// window slots. This kernel serves d_head 64 (d_head 128 runs on the tensor
+// cores, decode_tc.cu), and both sizes in the H2Share reuse step, whose
+// retrieval rows are borrowed positions gathered one row at a time.
 //
 // One CTA = one (sequence b, KV head, split) work unit; a split is a
 // contiguous range of cache rows. All G query heads of the GQA group are
@@ -163,14 +164,43 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
       const size_t new_off = ((size_t)b * g.Hkv + kvh) * D;
       const uint8_t* kn = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.k_new) + new_off);
       const uint8_t* vn = reinterpret_cast<const uint8_t*>(static_cast<const bf16*>(a.v_new) + new_off);
-      if (xr >= lo && xr < hi && lane < D / 8) {
+      // H2Share reuse step: the rows of a retrieval item are borrowed cache rows
+      const bool indexed = a.idx != nullptr && kind == 0;
+      const int32_t* rowlist =
+          indexed ? a.idx + ((size_t)b * a.n_idx_groups + a.idx_map[hi_idx]) * a.top_k : nullptr;
+      if ((indexed ? lo == 0 : (xr >= lo && xr < hi)) && lane < D / 8) {
         // append the new token (its row is read from the input below)
         reinterpret_cast<uint4*>(const_cast<uint8_t*>(Kc) + (size_t)xr * RB)[lane] =
             reinterpret_cast<const uint4*>(kn)[lane];
         reinterpret_cast<uint4*>(const_cast<uint8_t*>(Vc) + (size_t)xr * RB)[lane] =
             reinterpret_cast<const uint4*>(vn)[lane];
       }
-      if (lane == 0) {
+      if (indexed) {
+        // one 1D bulk copy per borrowed row, spread over the warp; indices are
+        // clamped to the rows held, so a bad list cannot read out of bounds
+        for (int row0 = lo; row0 < hi; row0 += TOK, ++it) {
+          const int st = it % NST;
+          int ok = 1;
+          if (lane == 0) {
+            ok = !*abort_flag;
+            if (ok && it >= NST && !mbar_wait(&empty[st], ((it / NST) & 1) ^ 1, a.err)) {
+              *abort_flag = 1;
+              ok = 0;
+            }
+          }
+          if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+          const int cnt = min(TOK, hi - row0);
+          if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)cnt * RB * 2);
+          __syncwarp();
+          uint8_t* ks = smem + st * C::STAGE_BYTES;
+          for (int r = lane; r < cnt; r += 32) {
+            const int cr = min(max(__ldg(rowlist + row0 + r), 0), t);
+            bulk_g2s(ks + (size_t)r * RB, cr == xr ? kn : Kc + (size_t)cr * RB, RB, &full[st]);
+            bulk_g2s(ks + (size_t)(TOK + r) * RB, cr == xr ? vn : Vc + (size_t)cr * RB, RB, &full[st]);
+          }
+          __syncwarp();
+        }
+      } else if (lane == 0) {
         for (int row0 = lo; row0 < hi && !*abort_flag; row0 += TOK, ++it) {
           const int st = it % NST;
           if (it >= NST && !mbar_wait(&empty[st], ((it / NST) & 1) ^ 1, a.err)) {
@@ -185,6 +215,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
         }
       }
       __syncwarp();
+      it = __shfl_sync(0xffffffffu, it, 0);  // lane 0 alone advanced it on a contiguous item
     }
     // every issued copy lands before the CTA can exit
     if (lane == 0)
@@ -428,15 +459,23 @@ cudaError_t launch_cfg(const DecodeArgs& a, cudaStream_t s) {
 
 }  // namespace
 
+bool decode_cc_supported(int D, int G) {
+  return (D == 64 || D == 128) && (G == 1 || G == 2 || G == 4 || G == 7 || G == 8);
+}
+
 bool decode_supported(int D, int G) {
   if (D == 128) return decode_uses_tc(D, G);
-  return D == 64 && (G == 1 || G == 2 || G == 4 || G == 7 || G == 8);
+  return decode_cc_supported(D, G);
 }
 
 // Two CTAs fit on an SM (about 100 KB of shared memory each), so 2 x SMs
 // CTAs run as one wave; small launches use fewer, at least 256 rows each.
 int decode_ctas(long long total_rows, int num_sms, int D, int G) {
   if (decode_uses_tc(D, G)) return decode_tc_ctas(total_rows, num_sms);
+  return decode_cc_ctas(total_rows, num_sms);
+}
+
+int decode_cc_ctas(long long total_rows, int num_sms) {
   const long long by_rows = (total_rows + 255) / 256;
   long long p = 2LL * num_sms;
   if (by_rows < p) p = by_rows;
@@ -445,10 +484,17 @@ int decode_ctas(long long total_rows, int num_sms, int D, int G) {
 
 size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 4 * dec::partial_stride(G, D); }
 
-cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
+cudaError_t launch_decode_cc(const DecodeArgs& a, cudaStream_t s) {
   const int D = a.geom.D, G = a.geom.G;
-  if (decode_uses_tc(D, G)) return launch_decode_tc(a, s);
-  if (D == 64) {
+  if (D == 128) {
+    switch (G) {
+      case 1: return launch_cfg<128, 1>(a, s);
+      case 2: return launch_cfg<128, 2>(a, s);
+      case 4: return launch_cfg<128, 4>(a, s);
+      case 7: return launch_cfg<128, 7>(a, s);
+      case 8: return launch_cfg<128, 8>(a, s);
+    }
+  } else if (D == 64) {
     switch (G) {
       case 1: return launch_cfg<64, 1>(a, s);
       case 2: return launch_cfg<64, 2>(a, s);
@@ -458,6 +504,11 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
     }
   }
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s) {
+  if (decode_uses_tc(a.geom.D, a.geom.G)) return launch_decode_tc(a, s);
+  return launch_decode_cc(a, s);
 }
 
 }  // namespace aoh

@@ -19,14 +19,16 @@ namespace dec {
 
 constexpr int kGroup = 16;  // parts merged per first-level group
 
-// Rows of item `id`. Retrieval: t + 1 rows; streaming: min(t + 1, S + W)
-// ring rows; t = tokens held before this step.
+// Rows of item `id`. Retrieval: t + 1 rows (min(top_k, t + 1) borrowed rows
+// in the H2Share reuse step); streaming: min(t + 1, S + W) ring rows;
+// t = tokens held before this step.
 __device__ __forceinline__ int item_rows(const DecodeArgs& a, int id) {
   const CacheGeom& g = a.geom;
   const int HK = g.n_r + g.n_s;
   const int b = id / HK, k = id - b * HK;
   const int t = __ldcg(&a.lens[b]);
-  return k < g.n_r ? t + 1 : min(t + 1, g.S + g.W);
+  if (k < g.n_r) return a.idx ? min(a.top_k, t + 1) : t + 1;
+  return min(t + 1, g.S + g.W);
 }
 
 // CTA whose row range contains global row x.
@@ -97,8 +99,9 @@ __device__ __forceinline__ float* partial_slot(const DecodeArgs& a, int q, int s
 }
 
 // Merge n partial states (part(j) returns the j-th) with log-sum-exp
-// weights. Writes the normalised bf16 output to `out`, or the merged partial
-// to `dst`. Run by NT threads that share named barrier 1. The partials sit
+// weights. Writes the normalised bf16 output to `out` (and, if `stats` is
+// given, the merged (max, sum) of every head to stats[0..G)), or the merged
+// partial to `dst`. Run by NT threads that share named barrier 1. The partials sit
 // in L2, so the merge is a chain of L2 round trips at the end of the launch.
 //
 // WIDE = false (few registers): m and l are staged in `scratch` (2*n*G + 2*G
@@ -107,7 +110,8 @@ __device__ __forceinline__ float* partial_slot(const DecodeArgs& a, int q, int s
 // U parts costs one round trip (O, m and l of all U parts loaded together)
 // and folds into a running per-element max, as in the online softmax.
 template <int G, int D, int NT, bool WIDE, class PartFn>
-__device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch) {
+__device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* out, float* dst, float* scratch,
+                                            float2* stats = nullptr) {
   if constexpr (!WIDE) {
     float* wts = scratch;          // [n][G] m, then the weights
     float* ls = scratch + n * G;   // [n][G] l
@@ -141,6 +145,7 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
       for (int j = 0; j < n; ++j) O += wts[j * G + r] * __ldcg(part(j) + idx);
       if (out) {
         out[idx] = __float2bfloat16_rn(O / Ls[r]);
+        if (stats && idx - r * D == 0) stats[r] = make_float2(Ms[r], Ls[r]);
       } else {
         __stcg(dst + idx, O);
         if (idx - r * D == 0) {
@@ -212,6 +217,7 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
         w.x = float2_to_bf16x2(O[e].x * inv, O[e].y * inv);
         w.y = float2_to_bf16x2(O[e].z * inv, O[e].w * inv);
         *reinterpret_cast<uint2*>(out + idx) = w;
+        if (stats && idx - r * D == 0) stats[r] = make_float2(M[e], L[e]);
       } else {
         __stcg(reinterpret_cast<float4*>(dst + idx), O[e]);
         if (idx - r * D == 0) {
@@ -233,7 +239,8 @@ __device__ __forceinline__ void merge_parts(int n, PartFn part, __nv_bfloat16* o
 // of shared memory, `scratch` as for merge_parts.
 template <int G, int D, int NT, bool WIDE>
 __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, int lst, int id,
-                                           __nv_bfloat16* outp, float* scratch, volatile int* flag) {
+                                           __nv_bfloat16* outp, float* scratch, volatile int* flag,
+                                           float2* stats = nullptr) {
   // the barrier orders every thread's partial stores before thread 0's fence
   // and counter update (release); thread 0's fence after a last arrival
   // orders the other parts' stores before the loads below (acquire)
@@ -260,7 +267,7 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
     return partial_slot(a, q, q == f ? 1 : 0, G, D);
   };
   if (n_groups == 1) {
-    merge_parts<G, D, NT, WIDE>(gsz, own, outp, nullptr, scratch);
+    merge_parts<G, D, NT, WIDE>(gsz, own, outp, nullptr, scratch, stats);
     return;
   }
   merge_parts<G, D, NT, WIDE>(gsz, own, nullptr, partial_slot(a, p0, 2 + gslot, G, D), scratch);
@@ -280,7 +287,7 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
     const int q = f + j * kGroup;
     return partial_slot(a, q, 2 + (q == f ? 1 : 0), G, D);
   };
-  merge_parts<G, D, NT, WIDE>(n_groups, grp_part, outp, nullptr, scratch);
+  merge_parts<G, D, NT, WIDE>(n_groups, grp_part, outp, nullptr, scratch, stats);
 }
 
 // The launch's last CTA advances every sequence length by one. Called by

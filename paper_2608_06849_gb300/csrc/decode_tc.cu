@@ -338,6 +338,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
         float s[G];
 #pragma unroll
         for (int h = 0; h < G; ++h) s[h] = valid ? __uint_as_float(v[h]) * a.scale_log2 : -INFINITY;
+        if (a.scores != nullptr && !strm && valid) {
+          // H2Share anchor step: this row's scores for the top-k selection
+          float* sc = a.scores + ((size_t)(b * g.n_r + k) * G) * a.score_stride + row0 + t;
+#pragma unroll
+          for (int h = 0; h < G; ++h) sc[(size_t)h * a.score_stride] = s[h];
+        }
 
         // per-head maximum over the tile: each warp, then the four warps
         float* rx = red + x * 64;
@@ -432,9 +438,19 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
 
       const int f = dec::cta_of(item_off, total, P), lst = dec::cta_of(item_off + rows - 1, total, P);
       bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * kD;
+      float2* st = (a.scores != nullptr && !strm) ? a.score_stats + (size_t)(b * g.n_r + k) * G : nullptr;
       if (f == lst) {
 #pragma unroll
         for (int h = 0; h < G; ++h) outp[h * kD + t] = __float2bfloat16_rn(__uint_as_float(o[h]) / L[h]);
+        if (st != nullptr && t < G) {
+          float mt = m[0], lt = L[0];
+#pragma unroll
+          for (int h = 1; h < G; ++h) {
+            mt = (t == h) ? m[h] : mt;
+            lt = (t == h) ? L[h] : lt;
+          }
+          st[t] = make_float2(mt, lt);
+        }
       } else {
         float* pbase = dec::partial_slot(a, p, p == f ? 1 : 0, G, kD);
 #pragma unroll
@@ -449,7 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
           __stcg(pbase + G * kD + t, mt);
           __stcg(pbase + G * kD + G + t, lt);
         }
-        dec::merge_item<G, kD, kSoftmaxThreads, true>(a, p, f, lst, id, outp, ms, sh32 + 1);
+        dec::merge_item<G, kD, kSoftmaxThreads, true>(a, p, f, lst, id, outp, ms, sh32 + 1, st);
       }
       named_barrier_sync(1, kSoftmaxThreads);
     }

@@ -59,6 +59,20 @@ struct DecodeArgs {
   uint32_t* err;      // error word
   int n_ctas;         // CTAs sharing the rows of all items equally
   float scale_log2;   // log2(e) / sqrt(D)
+  // H2Share anchor step (tcgen05 kernel): when non-null, every retrieval row's
+  // scores (log2 units) go to scores[((b * n_r + i) * G + h) * score_stride + row],
+  // and each retrieval head's final softmax state (max, sum of 2^(s - max))
+  // to score_stats[(b * n_r + i) * G + h].
+  float* scores = nullptr;
+  int score_stride = 0;
+  float2* score_stats = nullptr;
+  // H2Share reuse step (CUDA-core kernel): when non-null, retrieval item
+  // (b, i) attends only to the cache rows idx[(b * n_idx_groups + idx_map[i]) *
+  // top_k + r], r < min(top_k, t + 1).
+  const int32_t* idx = nullptr;
+  int top_k = 0;
+  int n_idx_groups = 0;
+  uint8_t idx_map[kMaxKvHeads] = {};
 };
 
 struct AppendArgs {
@@ -99,6 +113,22 @@ bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv);
 bool make_cache_region_maps(CUtensorMap* tcr, CUtensorMap* tcs, const CacheGeom& g, const void* kv);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
+// The CUDA-core decode kernel for any supported (D, G) (the H2Share reuse
+// step takes this path at d_head 128 too), with its CTA count.
+cudaError_t launch_decode_cc(const DecodeArgs& a, cudaStream_t s);
+int decode_cc_ctas(long long total_rows, int num_sms);
+bool decode_cc_supported(int D, int G);
+// H2Share anchor selection after a decode step that wrote its scores to
+// the start of `ws` ([B][n_r][G][max_seq] floats): per (sequence, retrieval
+// head) the top_k positions by group importance. `ws` holds
+// h2_workspace_floats() floats.
+size_t h2_workspace_floats(int B, int n_r, int G, int max_seq);
+// Where the decode kernel writes the scores and per-head states in `ws`.
+void h2_decode_outputs(float* ws, int B, int n_r, int G, int max_seq, float** scores, float2** stats);
+// Zero the histograms of a new workspace (the select kernel keeps them zero).
+cudaError_t h2_workspace_clear(float* ws, int B, int n_r, int G, int max_seq, cudaStream_t s);
+cudaError_t launch_h2_topk(float* ws, int max_seq, const int32_t* lens, int B, int n_r, int G, int top_k,
+                           int32_t* idx_out, cudaStream_t s);
 // CTAs for a decode launch over `total_rows` cached rows on `num_sms` SMs
 // (the kernel is chosen by D and G).
 int decode_ctas(long long total_rows, int num_sms, int D, int G);

@@ -26,3 +26,17 @@ def test_attended_pairs_chunk_rule(T, S, W, K):
     for streaming in (False, True):
         m = oatt.allowed_mask(np.arange(T), np.arange(T), streaming, S, W, K)
         assert bench.attended_pairs_chunk(T, S, W, K, streaming) == int(m.sum())
+
+
+def test_reuse_bytes_reduce_to_decode_bytes():
+    """With top_k covering every row, a reuse step moves the decode step's
+    bytes plus its index lists (4 bytes per borrowed row)."""
+    from paper_2608_06849_gb300.workloads import DECODE_128K, labels_for
+    wl = DECODE_128K
+    labels = labels_for(wl)
+    lens = [1000, 37, 5000]
+    n_r = sum(1 for x in labels if x == 0)
+    big = bench.reuse_bytes(lens, labels, wl, 10 ** 9)
+    assert big == bench.decode_bytes(lens, labels, wl) + 4 * n_r * sum(t + 1 for t in lens)
+    small = bench.reuse_bytes(lens, labels, wl, 8)
+    assert small < big

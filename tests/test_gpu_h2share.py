@@ -1,0 +1,201 @@
+"""H2Share on the GPU (the paper's H2Share section, GQA extension appendix)
+against the oracle on the same bf16 inputs.
+
+Anchor step: the decode output as in every decode test; the selected
+positions form a valid top-k set of the oracle's float64 importance. The
+GPU ranks fp32 scores, so positions whose importance lies within the fp32
+error of the k-th value may legitimately differ: every selected position
+must be at least the k-th importance and every other at most it, each up
+to that error (1e-4 relative). Reuse step: retrieval groups against the
+oracle's sparse attention over the given positions (the lists the anchor
+produced, or synthetic lists), streaming groups against the decode step;
+the cache image is checked bit-exactly.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_cases import assert_matches, check_cache_image, ensure_lib, f64
+from oracle import attention as oatt
+from oracle import h2share as ohs
+from paper_2608_06849_gb300 import aoh
+from paper_2608_06849_gb300.workloads import Workload, decode_inputs, randn_bf16
+
+pytestmark = pytest.mark.gpu
+REL = 1e-4
+
+
+def _filled_cache(B, Hq, Hkv, D, T, S, W, labels, steps, seed):
+    cache = aoh.Cache(B, Hq, Hkv, D, T + steps, S, W, labels)
+    k = randn_bf16((B, T, Hkv, D), seed + 1, "cuda")
+    v = randn_bf16((B, T, Hkv, D), seed + 2, "cuda")
+    k[:, 0] *= 8
+    cache.prefill(None, k, v, None)
+    torch.cuda.synchronize()
+    return cache, k, v
+
+
+def _check_selection(sel, imp, k):
+    n = imp.shape[0]
+    m = min(k, n)
+    assert np.all(sel[m:] == -1)
+    s = sel[:m]
+    assert np.all(np.diff(s) > 0) and s.min() >= 0 and s.max() < n
+    if m == n:
+        return
+    thr = np.sort(imp)[::-1][m - 1]
+    tol = REL * thr + 1e-12
+    rest = np.setdiff1d(np.arange(n), s)
+    assert imp[s].min() >= thr - tol, (imp[s].min(), thr)
+    assert imp[rest].max() <= thr + tol, (imp[rest].max(), thr)
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,T,labels,top_k", [
+    (2, 8, 2, 700, [0, 1], 64),
+    (1, 14, 2, 1500, [0, 0], 300),
+    (2, 16, 4, 257, [0, 1, 0, 1], 1000),      # top_k beyond the rows held
+    (1, 8, 2, 4000, [0, 0], 1),
+])
+def test_anchor_step_selects_top_k(B, Hq, Hkv, T, labels, top_k):
+    ensure_lib()
+    D, S, W, steps = 128, 4, 64, 2
+    g = Hq // Hkv
+    cache, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, steps, 31)
+    wl = Workload("anchor", B, Hq, Hkv, D, T, steps, S, W, sum(labels), seed=4)
+    retr = [h for h in range(Hkv) if labels[h] == 0]
+    kall = [f64(k[b]) for b in range(B)]
+    vall = [f64(v[b]) for b in range(B)]
+    for step in range(steps):
+        dq, dk, dv = decode_inputs(wl, step, device="cuda")
+        out = torch.full_like(dq, float("nan"))
+        idx = torch.full((B, len(retr), top_k), -7, dtype=torch.int32, device="cuda")
+        cache.decode_step_anchor(dq, dk, dv, out, top_k, idx)
+        torch.cuda.synchronize()
+        sel = idx.cpu().numpy()
+        for b in range(B):
+            kall[b] = np.concatenate([kall[b], f64(dk[b])[None]])
+            vall[b] = np.concatenate([vall[b], f64(dv[b])[None]])
+            qb = f64(dq[b])
+            want = oatt.decode_step(qb, kall[b], vall[b], labels, S, W)
+            mag = oatt.decode_step(qb, kall[b], np.abs(vall[b]), labels, S, W)
+            assert_matches(f64(out[b]), want, f"anchor decode {step} b={b}", mag)
+            for i, kvh in enumerate(retr):
+                imp = ohs.group_importance(qb[kvh * g:(kvh + 1) * g], kall[b][:, kvh])
+                _check_selection(sel[b, i], imp, top_k)
+    cache.check()
+    cache.close()
+
+
+def _reuse_case(B, Hq, Hkv, D, T, S, W, labels, top_k, n_anchor, group_map, steps=2, seed=41):
+    ensure_lib()
+    g = Hq // Hkv
+    cache, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, steps, seed)
+    wl = Workload("reuse", B, Hq, Hkv, D, T, steps, S, W, sum(labels), seed=6)
+    retr = [h for h in range(Hkv) if labels[h] == 0]
+    rng = np.random.default_rng(seed)
+    kall = [f64(k[b]) for b in range(B)]
+    vall = [f64(v[b]) for b in range(B)]
+    ktn = [k[b].cpu() for b in range(B)]
+    vtn = [v[b].cpu() for b in range(B)]
+    for step in range(steps):
+        t = T + step                       # the new token's position
+        lists = np.full((B, n_anchor, top_k), -1, dtype=np.int32)
+        for b in range(B):
+            for a in range(n_anchor):
+                m = min(top_k, t + 1)
+                pick = rng.choice(t + 1, size=m, replace=False)
+                if a == 0 and m < t + 1:
+                    pick[0] = t            # the new token among the borrowed rows
+                    pick = np.unique(pick)
+                    while len(pick) < m:
+                        pick = np.unique(np.concatenate([pick, rng.choice(t, size=m - len(pick))]))
+                lists[b, a, :m] = np.sort(pick)[:m]
+        idx = torch.from_numpy(lists).cuda()
+        dq, dk, dv = decode_inputs(wl, step, device="cuda")
+        out = torch.full_like(dq, float("nan"))
+        cache.decode_step_reuse(dq, dk, dv, out, idx, top_k, group_map)
+        torch.cuda.synchronize()
+        for b in range(B):
+            kall[b] = np.concatenate([kall[b], f64(dk[b])[None]])
+            vall[b] = np.concatenate([vall[b], f64(dv[b])[None]])
+            ktn[b] = torch.cat([ktn[b], dk[b][None].cpu()])
+            vtn[b] = torch.cat([vtn[b], dv[b][None].cpu()])
+            qb = f64(dq[b])
+            full = oatt.decode_step(qb, kall[b], vall[b], labels, S, W)
+            fmag = oatt.decode_step(qb, kall[b], np.abs(vall[b]), labels, S, W)
+            for kvh in range(Hkv):
+                hs = slice(kvh * g, (kvh + 1) * g)
+                if labels[kvh] == 0:
+                    pos = lists[b, group_map[retr.index(kvh)]]
+                    pos = pos[pos >= 0]
+                    want = ohs.sparse_attend(qb[hs], kall[b][:, kvh], vall[b][:, kvh], pos)
+                    mag = ohs.sparse_attend(qb[hs], kall[b][:, kvh], np.abs(vall[b][:, kvh]), pos)
+                else:
+                    want, mag = full[hs], fmag[hs]
+                assert_matches(f64(out[b, hs]), want, f"reuse step {step} b={b} kv={kvh}", mag)
+    cache.check()
+    assert cache.lens() == [T + steps] * B
+    kpad = torch.stack(ktn)
+    vpad = torch.stack(vtn)
+    check_cache_image(cache, kpad, vpad, [T + steps] * B, labels, S, W)
+    cache.close()
+
+
+@pytest.mark.parametrize("D,Hq,Hkv,labels,top_k,n_anchor,gmap", [
+    (128, 8, 2, [0, 1], 200, 3, [2]),
+    (128, 14, 2, [0, 0], 97, 2, [1, 0]),
+    (128, 16, 4, [0, 1, 0, 0], 5000, 1, [0, 0, 0]),   # every row borrowed: a full decode
+    (64, 16, 2, [1, 0], 33, 4, [3]),
+])
+def test_reuse_step_attends_to_borrowed_rows(D, Hq, Hkv, labels, top_k, n_anchor, gmap):
+    _reuse_case(2, Hq, Hkv, D, 900, 4, 50, labels, top_k, n_anchor, gmap)
+
+
+def test_anchor_then_reuse():
+    """An anchor layer and a reuse layer of one block at the same step: the
+    reuse layer attends to its own K/V at the positions the anchor chose."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, top_k = 2, 8, 2, 128, 1200, 4, 64, 128
+    labels = [0, 1]
+    g = Hq // Hkv
+    anchor, _, _ = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, 1, 51)
+    reuse, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, 1, 61)
+    wa = Workload("a", B, Hq, Hkv, D, T, 1, S, W, 1, seed=7)
+    wr = Workload("r", B, Hq, Hkv, D, T, 1, S, W, 1, seed=8)
+    qa, ka, va = decode_inputs(wa, 0, device="cuda")
+    qr, kr, vr = decode_inputs(wr, 0, device="cuda")
+    idx = torch.empty((B, 1, top_k), dtype=torch.int32, device="cuda")
+    oa = torch.empty_like(qa)
+    orr = torch.empty_like(qr)
+    anchor.decode_step_anchor(qa, ka, va, oa, top_k, idx)
+    reuse.decode_step_reuse(qr, kr, vr, orr, idx, top_k, [0])
+    torch.cuda.synchronize()
+    sel = idx.cpu().numpy()
+    for b in range(B):
+        kk = np.concatenate([f64(k[b]), f64(kr[b])[None]])
+        vv = np.concatenate([f64(v[b]), f64(vr[b])[None]])
+        q = f64(qr[b])
+        want = ohs.sparse_attend(q[:g], kk[:, 0], vv[:, 0], sel[b, 0])
+        mag = ohs.sparse_attend(q[:g], kk[:, 0], np.abs(vv[:, 0]), sel[b, 0])
+        assert_matches(f64(orr[b, :g]), want, f"reuse after anchor b={b}", mag)
+        full = oatt.decode_step(q, kk, vv, labels, S, W)
+        assert_matches(f64(orr[b, g:]), full[g:], f"reuse streaming b={b}")
+    anchor.close()
+    reuse.close()
+
+
+def test_reuse_rejects_bad_maps():
+    ensure_lib()
+    cache, _, _ = _filled_cache(1, 8, 2, 128, 64, 4, 16, [0, 1], 1, 71)
+    q = torch.zeros(1, 8, 128, dtype=torch.bfloat16, device="cuda")
+    kv = torch.zeros(1, 2, 128, dtype=torch.bfloat16, device="cuda")
+    idx = torch.zeros((1, 2, 8), dtype=torch.int32, device="cuda")
+    with pytest.raises(aoh.AohError) as e:
+        cache.decode_step_reuse(q, kv, kv, torch.empty_like(q), idx, 8, [2])
+    assert e.value.status == 1
+    with pytest.raises(aoh.AohError) as e:
+        cache.decode_step_anchor(q, kv, kv, torch.empty_like(q), 0, idx)
+    assert e.value.status == 1
+    assert cache.lens() == [64]
+    cache.close()
