@@ -215,6 +215,17 @@ aoh_status aoh_cache_reset(aoh_cache* cache, void* stream);
  */
 aoh_status aoh_cache_check(aoh_cache* cache, void* stream);
 
+/*
+ * Self-test of the bounded waits every kernel uses (the paper has no
+ * counterpart): one warp waits on a barrier that nothing arrives at for
+ * limit_ns (1 ms .. 2 s), gives up, and records the timeout in the cache's
+ * error word, as a kernel whose partner role stalled would. The next
+ * aoh_cache_check returns AOH_ERR_TIMEOUT (and clears the word); the cache
+ * and the CUDA context stay usable. *elapsed_ns (may be NULL) receives how
+ * long the wait lasted. Synchronises `stream`. Errors: INVALID, CUDA.
+ */
+aoh_status aoh_cache_selftest_wait(aoh_cache* cache, int64_t limit_ns, int64_t* elapsed_ns, void* stream);
+
 /* Release the handle and its device metadata (not the KV buffer). NULL is a no-op. */
 void aoh_cache_destroy(aoh_cache* cache);
 

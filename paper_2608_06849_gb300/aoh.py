@@ -38,6 +38,7 @@ EXPORTS = [
     "aoh_classify",
     "aoh_decode_step_anchor",
     "aoh_decode_step_reuse",
+    "aoh_cache_selftest_wait",
 ]
 
 
@@ -80,6 +81,7 @@ def load():
         "aoh_cache_region": (i32, [P, i32, i32, szp, szp, i32p]),
         "aoh_cache_reset": (i32, [P, P]),
         "aoh_cache_check": (i32, [P, P]),
+        "aoh_cache_selftest_wait": (i32, [P, ctypes.c_int64, ctypes.POINTER(ctypes.c_int64), P]),
         "aoh_cache_destroy": (None, [P]),
         "aoh_last_error": (ctypes.c_char_p, []),
         "aoh_version": (i32, []),
@@ -223,6 +225,13 @@ def aoh_cache_reset(cache, stream=None):
 
 def aoh_cache_check(cache, stream=None):
     _check(load().aoh_cache_check(cache, _stream_ptr(stream)))
+
+
+def aoh_cache_selftest_wait(cache, limit_ns, stream=None):
+    """Run the bounded-wait self-test; returns the wait's duration in ns."""
+    el = ctypes.c_int64()
+    _check(load().aoh_cache_selftest_wait(cache, int(limit_ns), ctypes.byref(el), _stream_ptr(stream)))
+    return el.value
 
 
 def aoh_cache_destroy(cache):

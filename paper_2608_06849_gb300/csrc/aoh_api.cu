@@ -273,6 +273,23 @@ aoh_status aoh_cache_check(aoh_cache* cache, void* stream) {
   return AOH_OK;
 }
 
+aoh_status aoh_cache_selftest_wait(aoh_cache* cache, int64_t limit_ns, int64_t* elapsed_ns, void* stream) {
+  if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
+  if (limit_ns < 1000000 || limit_ns > 2000000000LL)
+    return fail(AOH_ERR_INVALID, "limit_ns must be in [1 ms, 2 s]");
+  cudaStream_t s = (cudaStream_t)stream;
+  // the elapsed time is staged in the metadata block's spare word after the error word
+  unsigned long long* d_elapsed = reinterpret_cast<unsigned long long*>(cache->d_err + 8);
+  cudaError_t e = launch_wait_selftest(cache->d_err, (uint64_t)limit_ns, d_elapsed, s);
+  if (e != cudaSuccess) return cuda_fail(e, "self-test kernel launch");
+  unsigned long long el = 0;
+  e = cudaMemcpyAsync(&el, d_elapsed, sizeof(el), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "self-test read back");
+  if (elapsed_ns) *elapsed_ns = (int64_t)el;
+  return AOH_OK;
+}
+
 aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, const int32_t* seq_lens,
                        aoh_cache* cache, void* out, void* stream) {
   if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");

@@ -73,14 +73,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
 }
 
 // As mbar_wait, but also gives up (without touching *err) once another role
-// of the CTA has raised *abort_flag; a timeout raises it.
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_t* err, volatile int* abort_flag) {
+// of the CTA has raised *abort_flag; a timeout raises it. `limit_ns` bounds
+// the wait (kWaitLimitNs in the kernels; shorter in the self-test).
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_t* err, volatile int* abort_flag,
+                                         uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       atomicOr(err, kErrTimeout);
       *abort_flag = 1;
       return false;

@@ -101,6 +101,11 @@ struct PrefillTcArgs {
   float scale_log2;
 };
 
+// One warp waits on an mbarrier nothing arrives at, for limit_ns; the timeout
+// lands in *err; *elapsed_ns receives how long the wait lasted (0 if it did
+// not give up).
+cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns, unsigned long long* elapsed_ns, cudaStream_t s);
+
 // Store `msg` as the calling thread's aoh_last_error() message.
 void record_error(const char* msg);
 
