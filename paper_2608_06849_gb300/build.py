@@ -34,9 +34,9 @@ def source_digest():
 
 
 KERNEL_SOURCES = {
-    "decode": ["decode.cu", "decode_common.cuh", "common.cuh"],
-    "decode_tc": ["decode_tc.cu", "decode_common.cuh", "tc.cuh", "common.cuh"],
-    "prefill": ["prefill_tc.cu", "tc.cuh", "common.cuh"],
+    "decode": ["decode.cu", "decode_common.cuh", "common.cuh", "internal.h"],
+    "decode_tc": ["decode_tc.cu", "decode_common.cuh", "tc.cuh", "common.cuh", "internal.h"],
+    "prefill": ["prefill_tc.cu", "tc.cuh", "common.cuh", "internal.h"],
 }
 
 
