@@ -132,3 +132,65 @@ def test_stack_256k_one_layer_sampled():
     assert total == 28 * (2 * (T + wl.decode_steps) + 2 * (wl.sink + wl.window)) * wl.d_head * 4
     assert full / total > 1.96
     cache.close()
+
+
+def test_h2share_at_decode_128k_sampled():
+    """H2Share at the size bench.py times it (Llama-3-8B shape, B=16, 128K
+    cached tokens, top_k 2048): one anchor step, then one reuse step on the
+    same cache borrowing the anchor's positions. Sampled sequences: the
+    anchor's selections form a valid top-k set of the oracle's importance
+    (up to fp32 score error) and its outputs match the decode step; the reuse
+    outputs match the oracle's attention over the borrowed positions."""
+    from oracle import h2share as ohs
+    wl = DECODE_128K
+    ensure_lib()
+    labels = labels_for(wl)
+    B, T, D, g = wl.batch, wl.prefill_len, wl.d_head, wl.g
+    top_k = 2048
+    cache = aoh.Cache(B, wl.n_q_heads, wl.n_kv_heads, D, T + 4, wl.sink, wl.window, labels)
+    kfill = randn_bf16((B, T, wl.n_kv_heads, D), 7001, "cuda")
+    vfill = randn_bf16((B, T, wl.n_kv_heads, D), 7002, "cuda")
+    cache.prefill(None, kfill, vfill, None)
+    retr = [h for h in range(wl.n_kv_heads) if labels[h] == 0]
+    idx = torch.full((B, len(retr), top_k), -7, dtype=torch.int32, device="cuda")
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    out = torch.full_like(dq, float("nan"))
+    cache.decode_step_anchor(dq, dk, dv, out, top_k, idx)
+    rq, rk, rv = decode_inputs(wl, 1, device="cuda")
+    rout = torch.full_like(rq, float("nan"))
+    cache.decode_step_reuse(rq, rk, rv, rout, idx, top_k, list(range(len(retr))))
+    torch.cuda.synchronize()
+    cache.check()
+    sel = idx.cpu().numpy()
+    for b in (0, 9, 15):
+        kk = np.concatenate([f64(kfill[b]), f64(dk[b])[None]])
+        vv = np.concatenate([f64(vfill[b]), f64(dv[b])[None]])
+        q = f64(dq[b])
+        for i, kv in enumerate(retr):
+            hs = slice(kv * g, (kv + 1) * g)
+            imp = ohs.group_importance(q[hs], kk[:, kv])
+            s = sel[b, i]
+            assert np.all(np.diff(s) > 0) and s.min() >= 0 and s.max() <= T and len(s) == top_k
+            thr = np.sort(imp)[::-1][top_k - 1]
+            rest = np.setdiff1d(np.arange(T + 1), s)
+            assert imp[s].min() >= thr * (1 - 1e-4) and imp[rest].max() <= thr * (1 + 1e-4)
+            want = oatt.decode_step(q[hs], kk[:, kv:kv + 1], vv[:, kv:kv + 1], [0], wl.sink, wl.window)
+            mag = oatt.decode_step(q[hs], kk[:, kv:kv + 1], np.abs(vv[:, kv:kv + 1]), [0], wl.sink, wl.window)
+            assert_matches(f64(out[b, hs]), want, f"anchor b={b} kv={kv}", mag)
+        # reuse step at position T + 1: its own new K/V appended after the anchor's
+        kr = np.concatenate([kk, f64(rk[b])[None]])
+        vr = np.concatenate([vv, f64(rv[b])[None]])
+        qr = f64(rq[b])
+        for i, kv in enumerate(retr):
+            hs = slice(kv * g, (kv + 1) * g)
+            pos = sel[b, i]
+            want = ohs.sparse_attend(qr[hs], kr[:, kv], vr[:, kv], pos)
+            mag = ohs.sparse_attend(qr[hs], kr[:, kv], np.abs(vr[:, kv]), pos)
+            assert_matches(f64(rout[b, hs]), want, f"reuse b={b} kv={kv}", mag)
+        for kv in range(wl.n_kv_heads):
+            if labels[kv] == 0:
+                continue
+            hs = slice(kv * g, (kv + 1) * g)
+            want = oatt.decode_step(qr[hs], kr[:, kv:kv + 1], vr[:, kv:kv + 1], [1], wl.sink, wl.window)
+            assert_matches(f64(rout[b, hs]), want, f"reuse streaming b={b} kv={kv}")
+    cache.close()
