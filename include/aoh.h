@@ -195,6 +195,36 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
                                  void* out, const int32_t* indices, int32_t n_anchor_groups, int32_t top_k,
                                  const int32_t* group_map, void* stream);
 
+/*
+ * H2Share head mapping (the paper's H2Share section, Eq. sim; GQA extension
+ * appendix), offline, from the frozen weights of an anchor layer and a reuse
+ * layer. sim(h, h') is the normalised Frobenius inner product of the two
+ * kernel matrices M = W_K^T W_Q, computed through traces of d_head x d_head
+ * products; a group-pair similarity is the mean over the query-head pairs;
+ * each reuse retrieval group maps to the anchor retrieval group of highest
+ * similarity (ties to the lower index).
+ *   w_q_*  device bf16 [n_q_heads][d_head][d_model]; w_k_* [n_kv_heads][...],
+ *          laid out as for aoh_classify; 16-byte aligned; d_model a
+ *          multiple of 8; d_head 64 or 128.
+ *   anchor_labels, reuse_labels  host uint8 [n_kv_heads] (AOH_RETRIEVAL /
+ *          AOH_STREAMING), e.g. from aoh_classify.
+ *   map_out        host int32 [n_kv_heads]: for each reuse group, the
+ *                  anchor group it borrows from; -1 for streaming reuse
+ *                  groups (or when the anchor layer has no retrieval group).
+ *                  Listing the retrieval entries in increasing reuse-group
+ *                  order, converted to anchor retrieval slots, gives the
+ *                  group_map of aoh_decode_step_reuse.
+ *   group_sim_out  host double [n_kv_heads][n_kv_heads] (anchor-major), or NULL.
+ * The d_model contractions run on the tensor cores (bf16 in, fp32
+ * accumulate); traces and norms in fp64. Allocates temporary device memory
+ * stream-ordered and synchronises `stream`. Errors: INVALID, UNSUPPORTED,
+ * TIMEOUT, CUDA.
+ */
+aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_anchor, const void* w_q_reuse,
+                           const void* w_k_reuse, int32_t n_q_heads, int32_t n_kv_heads, int32_t d_head,
+                           int32_t d_model, const uint8_t* anchor_labels, const uint8_t* reuse_labels,
+                           int32_t* map_out, double* group_sim_out, void* stream);
+
 /* Copy the host-side lengths (tokens held per sequence) into lens_out [B]. */
 aoh_status aoh_cache_lens(const aoh_cache* cache, int32_t* lens_out);
 

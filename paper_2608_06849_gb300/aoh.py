@@ -39,6 +39,7 @@ EXPORTS = [
     "aoh_decode_step_anchor",
     "aoh_decode_step_reuse",
     "aoh_cache_selftest_wait",
+    "aoh_h2share_map",
 ]
 
 
@@ -81,6 +82,8 @@ def load():
         "aoh_cache_region": (i32, [P, i32, i32, szp, szp, i32p]),
         "aoh_cache_reset": (i32, [P, P]),
         "aoh_cache_check": (i32, [P, P]),
+        "aoh_h2share_map": (i32, [P, P, P, P, i32, i32, i32, i32, u8p, u8p, i32p,
+                                  ctypes.POINTER(ctypes.c_double), P]),
         "aoh_cache_selftest_wait": (i32, [P, ctypes.c_int64, ctypes.POINTER(ctypes.c_int64), P]),
         "aoh_cache_destroy": (None, [P]),
         "aoh_last_error": (ctypes.c_char_p, []),
@@ -204,6 +207,39 @@ def aoh_classify(w_q, w_k, n_kv_heads, sparsity_pct, stream=None):
     labels = [list(lab[l * n_kv_heads:(l + 1) * n_kv_heads]) for l in range(L)]
     ers = [list(er[l * Hq:(l + 1) * Hq]) for l in range(L)]
     return (labels[0], ers[0]) if single else (labels, ers)
+
+
+def aoh_h2share_map(w_q_anchor, w_k_anchor, w_q_reuse, w_k_reuse, anchor_labels, reuse_labels, stream=None):
+    """Group mapping of a reuse layer onto an anchor layer. Weights: bf16 CUDA
+    tensors [Hq, d_head, d_model] / [Hkv, d_head, d_model]. Returns (map, sim):
+    map[r] = anchor group of reuse group r (-1 if streaming), sim [Hkv][Hkv]
+    anchor-major group similarities."""
+    Hq, dh, dm = w_q_anchor.shape
+    Hkv = w_k_anchor.shape[0]
+    mp = (ctypes.c_int32 * Hkv)()
+    sim = (ctypes.c_double * (Hkv * Hkv))()
+    _check(load().aoh_h2share_map(_ptr(w_q_anchor, "w_q_anchor"), _ptr(w_k_anchor, "w_k_anchor"),
+                                  _ptr(w_q_reuse, "w_q_reuse"), _ptr(w_k_reuse, "w_k_reuse"), Hq, Hkv, dh, dm,
+                                  _labels_arr(anchor_labels), _labels_arr(reuse_labels), mp, sim,
+                                  _stream_ptr(stream)))
+    return list(mp), [list(sim[a * Hkv:(a + 1) * Hkv]) for a in range(Hkv)]
+
+
+def reuse_group_map(head_map, anchor_labels, reuse_labels):
+    """The group_map of aoh_decode_step_reuse from a mapping head_map[r] =
+    anchor KV group (aoh_h2share_map): for each reuse retrieval group in
+    increasing order, the slot of its anchor group among the anchor's
+    retrieval groups (the order of the anchor step's index lists)."""
+    slots = {a: i for i, a in enumerate(h for h, l in enumerate(anchor_labels) if int(l) == 0)}
+    out = []
+    for r, l in enumerate(reuse_labels):
+        if int(l) != 0:
+            continue
+        a = int(head_map[r])
+        if a not in slots:
+            raise ValueError(f"reuse retrieval group {r} maps to {a}, not an anchor retrieval group")
+        out.append(slots[a])
+    return out
 
 
 def aoh_cache_lens(cache, batch):

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -105,6 +106,9 @@ struct PrefillTcArgs {
 // lands in *err; *elapsed_ns receives how long the wait lasted (0 if it did
 // not give up).
 cudaError_t launch_wait_selftest(uint32_t* err, uint64_t limit_ns, unsigned long long* elapsed_ns, cudaStream_t s);
+
+// cuTensorMapEncodeTiled from the driver (nullptr if unavailable).
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn();
 
 // Store `msg` as the calling thread's aoh_last_error() message.
 void record_error(const char* msg);

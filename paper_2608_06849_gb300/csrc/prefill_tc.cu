@@ -497,6 +497,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
+}  // namespace
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -509,6 +511,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   }
   return fn;
 }
+
+namespace {
 
 // 4D map over a [B][T][H][D] bf16 tensor, box [1][128][1][64], 128-byte swizzle.
 bool make_map(CUtensorMap* map, const void* base, int B, int T, int H, int D) {

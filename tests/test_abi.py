@@ -25,7 +25,7 @@ def lib():
 def declared_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    names = re.findall(r"\b(aoh_[a-z_]+)\s*\(", text)
+    names = re.findall(r"\b(aoh_[a-z0-9_]+)\s*\(", text)
     return sorted(set(names))
 
 
@@ -122,6 +122,18 @@ def test_classify_rejects_bad_arguments_on_host(lib):
     assert lib.aoh_classify(fake, fake, 1, 8, 2, 128, 512, 101, None, lab, None) == 1
     assert lib.aoh_classify(fake, fake, 1, 8, 2, 128, 512, 50, None, None, None) == 1
     assert lib.aoh_classify(fake, fake, 5000, 8, 8, 128, 512, 50, None, lab, None) == 1  # > 65535 matrices
+
+
+def test_h2share_map_rejects_bad_arguments_on_host(lib):
+    lab = (ctypes.c_uint8 * 2)(0, 1)
+    mp = (ctypes.c_int32 * 2)()
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced
+    assert lib.aoh_h2share_map(None, fake, fake, fake, 8, 2, 128, 512, lab, lab, mp, None, None) == 1
+    assert lib.aoh_h2share_map(fake, fake, fake, fake, 8, 3, 128, 512, lab, lab, mp, None, None) == 1
+    assert lib.aoh_h2share_map(fake, fake, fake, fake, 8, 2, 96, 512, lab, lab, mp, None, None) == 5
+    assert lib.aoh_h2share_map(fake, fake, fake, fake, 8, 2, 128, 500, lab, lab, mp, None, None) == 1
+    bad = (ctypes.c_uint8 * 2)(0, 2)
+    assert lib.aoh_h2share_map(fake, fake, fake, fake, 8, 2, 128, 512, bad, lab, mp, None, None) == 1
 
 
 def test_bad_label_rejected(lib):
