@@ -19,14 +19,22 @@ namespace dec {
 
 constexpr int kGroup = 16;  // parts merged per first-level group
 
+// Tokens held by sequence b before this step: from the kernel's shared
+// memory copy of the lengths when it has one (`lens_s`), else from global
+// memory. Under a saturated HBM stream even an L2 hit costs microseconds,
+// which at an item switch would stall the TMA ring.
+__device__ __forceinline__ int seq_len(const DecodeArgs& a, int b, const int* lens_s) {
+  return lens_s ? lens_s[b] : __ldcg(&a.lens[b]);
+}
+
 // Rows of item `id`. Retrieval: t + 1 rows (min(top_k, t + 1) borrowed rows
 // in the H2Share reuse step); streaming: min(t + 1, S + W) ring rows;
 // t = tokens held before this step.
-__device__ __forceinline__ int item_rows(const DecodeArgs& a, int id) {
+__device__ __forceinline__ int item_rows(const DecodeArgs& a, int id, const int* lens_s = nullptr) {
   const CacheGeom& g = a.geom;
   const int HK = g.n_r + g.n_s;
   const int b = id / HK, k = id - b * HK;
-  const int t = __ldcg(&a.lens[b]);
+  const int t = seq_len(a, b, lens_s);
   if (k < g.n_r) return a.idx ? min(a.top_k, t + 1) : t + 1;
   return min(t + 1, g.S + g.W);
 }
@@ -41,7 +49,8 @@ __device__ __forceinline__ int cta_of(long long x, long long total, int P) {
 // rows, sh64[1] = first row of the first item this CTA touches, sh32[0] =
 // that item. `wsum` is THREADS / 32 longs of scratch shared memory.
 template <int THREADS>
-__device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* wsum, long long* sh64, int* sh32) {
+__device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* wsum, long long* sh64, int* sh32,
+                                               const int* lens_s = nullptr) {
   constexpr int NW = THREADS / 32;
   const CacheGeom& g = a.geom;
   const int n_items = g.B * (g.n_r + g.n_s);
@@ -50,7 +59,7 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* w
   const int per = (n_items + THREADS - 1) / THREADS;
   const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
   long long mine = 0;
-  for (int id = i0; id < i1; ++id) mine += item_rows(a, id);
+  for (int id = i0; id < i1; ++id) mine += item_rows(a, id, lens_s);
   long long inc = mine;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -78,7 +87,7 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* w
   if (i0 < i1 && off <= start && start < off + mine) {
     int id = i0;
     while (true) {
-      const int r = item_rows(a, id);
+      const int r = item_rows(a, id, lens_s);
       if (start < off + r) break;
       off += r;
       ++id;

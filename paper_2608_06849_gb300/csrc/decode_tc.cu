@@ -65,7 +65,9 @@ constexpr int MS_FLOATS = 1024;               // merge scratch
 constexpr int OFF_BAR = OFF_MS + MS_FLOATS * 4;
 constexpr int NBAR = 2 * kNS + 2 + 2 + 2 + 2 + 1 + 1;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
-constexpr int SMEM = OFF_MISC + 64 + 1024;
+constexpr int kLensCap = 2048;                // sequence lengths mirrored in shared memory
+constexpr int OFF_LENS = OFF_MISC + 64;
+constexpr int SMEM = OFF_LENS + kLensCap * 4 + 1024;
 constexpr uint32_t IDESC_S = idesc_bf16(kBN, kN, false, false);
 constexpr uint32_t IDESC_PV = idesc_bf16(kD, kN, false, true);
 static_assert(SMEM <= 232448, "shared memory");
@@ -96,6 +98,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   long long* sh64 = reinterpret_cast<long long*>(smem + OFF_MISC + 8);  // [0] total, [1] first offset
   int* sh32 = reinterpret_cast<int*>(sh64 + 2);                         // [0] first item, [1] merge flag
+  int* lens_s = reinterpret_cast<int*>(smem + OFF_LENS);
 
   const CacheGeom& g = a.geom;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -137,7 +140,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   // is visible after this wait; the next step may then start its prologue
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  dec::find_cta_range<kThreads>(a, reinterpret_cast<long long*>(sKV), sh64, sh32);
+  // the lengths cannot change during the launch (the last CTA to finish
+  // advances them), so every role reads this copy
+  const int* ls = g.B <= kLensCap ? lens_s : nullptr;
+  if (ls != nullptr) {
+    for (int i = threadIdx.x; i < g.B; i += kThreads) lens_s[i] = __ldcg(&a.lens[i]);
+    __syncthreads();
+  }
+  dec::find_cta_range<kThreads>(a, reinterpret_cast<long long*>(sKV), sh64, sh32, ls);
   __syncthreads();
   const long long total = sh64[0];
   const long long start = (long long)p * total / P;
@@ -154,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       bool ok = true;
       long long off = first_off;
       for (int id = first_id; id < n_items && off < end && ok; ++id) {
-        const int rows = dec::item_rows(a, id);
+        const int rows = dec::item_rows(a, id, ls);
         const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
         off += rows;
         if (lo >= hi) continue;
@@ -221,17 +231,44 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       __syncwarp();
     };
 
+    // An item's global inputs (its G query rows; the new token's K and V
+    // row) are fetched into registers one item ahead: under the saturated
+    // HBM stream a plain load takes microseconds, which at an item switch
+    // would sit between this item's last P V and the next item's first S.
+    // Lane l holds 16-byte chunks l, l + 32, ... of the G x 128 query block
+    // (head c / 16, chunk c % 16); lanes 0-15 the new K row's chunks, lanes
+    // 16-31 the new V row's.
+    constexpr int QV = (G * 16 + 31) / 32;
+    uint4 qr[QV];
+    uint4 nvr;
+    const int ch = lane & 15;
+    auto kv_head_of = [&](int id) {
+      const int k = id % HK;
+      return k >= g.n_r ? (int)g.s_head[k - g.n_r] : (int)g.r_head[k];
+    };
+    auto fetch_inputs = [&](int id) {
+      const int b = id / HK, kvh = kv_head_of(id);
+      const bf16* qg = static_cast<const bf16*>(a.q) + ((size_t)b * g.Hq + (size_t)kvh * G) * kD;
+#pragma unroll
+      for (int i = 0; i < QV; ++i) {
+        const int c = lane + 32 * i;
+        if (c < G * 16) qr[i] = *reinterpret_cast<const uint4*>(qg + (size_t)(c >> 4) * kD + (c & 15) * 8);
+      }
+      const size_t new_off = ((size_t)b * g.Hkv + kvh) * kD + ch * 8;
+      nvr = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(lane < 16 ? a.k_new : a.v_new) + new_off);
+    };
+    if (first_id < n_items) fetch_inputs(first_id);
+
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
-      const int rows = dec::item_rows(a, id);
+      const int rows = dec::item_rows(a, id, ls);
       const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
       off += rows;
       if (lo >= hi) continue;
       const int b = id / HK, k = id - b * HK;
       const bool strm = k >= g.n_r;
       const int hi_idx = strm ? k - g.n_r : k;
-      const int kvh = strm ? g.s_head[hi_idx] : g.r_head[hi_idx];
-      const int t = __ldcg(&a.lens[b]);
+      const int t = dec::seq_len(a, b, ls);
       const int cap = strm ? g.S + g.W : g.max_seq;
       const int xr = strm ? (t < g.S ? t : g.S + (t - g.S) % g.W) : t;  // the new token's row
       bf16* Kc = static_cast<bf16*>(a.kv) + (strm ? g.s_region(b, hi_idx) : g.r_region(b, hi_idx));
@@ -241,21 +278,21 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       wait_ofree(item_k - 1);
       if (!ok) break;
       {
-        const bf16* qg = static_cast<const bf16*>(a.q) + ((size_t)b * g.Hq + (size_t)kvh * G) * kD;
         uint8_t* qs = sQ + (item_k & 1) * kOpBuf;
-        for (int c = lane; c < G * 16; c += 32) {  // 16-byte chunks: head c / 16, chunk c % 16
-          const int h = c >> 4, cc = c & 15;
-          const uint4 v = *reinterpret_cast<const uint4*>(qg + (size_t)h * kD + cc * 8);
-          *reinterpret_cast<uint4*>(qs + (cc >> 3) * (kN * 128) + h * 128 + (((cc & 7) ^ (h & 7)) << 4)) = v;
+#pragma unroll
+        for (int i = 0; i < QV; ++i) {
+          const int c = lane + 32 * i;
+          if (c < G * 16) {
+            const int h = c >> 4, cc = c & 15;
+            *reinterpret_cast<uint4*>(qs + (cc >> 3) * (kN * 128) + h * 128 + (((cc & 7) ^ (h & 7)) << 4)) = qr[i];
+          }
         }
         fence_proxy_async_smem();
         __syncwarp();
       }
-      // lanes 0-15 hold the new K row's 16-byte chunks, lanes 16-31 the V row's
-      const int ch = lane & 15;
-      const size_t new_off = ((size_t)b * g.Hkv + kvh) * kD + ch * 8;
-      const uint4 nv = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(lane < 16 ? a.k_new : a.v_new) +
-                                                       new_off);
+      const uint4 nv = nvr;
+      // the next item of this CTA's range starts at its row 0
+      if (off < end && id + 1 < n_items) fetch_inputs(id + 1);
 
       for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
         const int st = it % kNS;
@@ -290,6 +327,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
         pend = Pend{it, st, item_k, row0 == lo};
         has_pend = true;
       }
+      // Inside an item, P(j) V(j) waits behind S(j + 1) so that the softmax
+      // of tile j + 1 can start meanwhile. At the item's end nothing can
+      // use the next item's S before this item's O is final, and holding
+      // P V back until the next item's first tile lands (a loaded-DRAM
+      // round trip) would hold the epilogue and this tile's ring slot.
+      if (has_pend && ok) {
+        issue_pv(pend);
+        has_pend = false;
+      }
       ++item_k;
     }
     if (has_pend) issue_pv(pend);
@@ -308,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
     bool ok = true, local_ok = true;
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
-      const int rows = dec::item_rows(a, id);
+      const int rows = dec::item_rows(a, id, ls);
       const long long item_off = off;
       const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
       off += rows;

@@ -107,6 +107,9 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // the next launch on the stream (the query side after the key side) may
+  // start its main loop now; it waits for this grid only before its epilogue
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     if (lane == 0) {
@@ -147,6 +150,8 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
     const int q4 = warp & 3;
     const bool ok = __all_sync(0xffffffffu, wait_bar(done, 0, a.err, abort_flag));
     const int row0 = tm * kTM + q4 * 32;
+    // trace mode reads the key-side matrices of the previous launch
+    if (a.trace) asm volatile("griddepcontrol.wait;" ::: "memory");
     if (ok && row0 < P.M) {
       tc_fence_after();
       const int r = row0 + lane;
@@ -218,6 +223,8 @@ bool add_problem(GemmArgs& g, const void* A, int M, const void* B, int N, int K,
   return true;
 }
 
+// A trace-mode launch overlaps the key-side launch before it (programmatic
+// dependent launch): only its epilogue waits for that grid.
 cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
@@ -227,8 +234,17 @@ cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s) {
   }
   int grid = 0;
   for (int i = 0; i < g.n_problems; ++i) grid += g.p[i].tiles;
-  gemm_kernel<<<grid, kGemmThreads, GEMM_SMEM, s>>>(g);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = GEMM_SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g.trace ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_kernel, g);
 }
 
 struct Labels {
@@ -238,7 +254,8 @@ struct Labels {
 // Head-pair traces from the block partials (each a sum over its (d_head/32)^2
 // blocks in a fixed order), then the group means and the argmax. parts:
 // pn [Hq d_head / 32]^2 for the numerators, pa / pr the same shape with only
-// the diagonal head blocks used.
+// the diagonal head blocks used. fp64 divides and square roots are slow on
+// this part, so each phase spreads its items over the block's threads.
 __global__ void map_kernel(const double* pn, const double* pa, const double* pr, int Hq, int Hkv, int dh,
                            Labels lab, double* num, double* na, double* nr, double* gsim, int32_t* map) {
   const int nb = dh / 32, ld = Hq * nb, g = Hq / Hkv;
@@ -248,23 +265,24 @@ __global__ void map_kernel(const double* pn, const double* pa, const double* pr,
       for (int y = 0; y < nb; ++y) s += p[(size_t)(h * nb + x) * ld + hp * nb + y];
     return s;
   };
-  for (int id = threadIdx.x; id < Hq * Hq + 2 * Hq; id += blockDim.x) {
-    if (id < Hq * Hq)
-      num[id] = block_sum(pn, id / Hq, id % Hq);
-    else if (id < Hq * Hq + Hq)
-      na[id - Hq * Hq] = block_sum(pa, id - Hq * Hq, id - Hq * Hq);
+  for (int id = threadIdx.x; id < 2 * Hq; id += blockDim.x) {
+    if (id < Hq)
+      na[id] = block_sum(pa, id, id);
     else
-      nr[id - Hq * Hq - Hq] = block_sum(pr, id - Hq * Hq - Hq, id - Hq * Hq - Hq);
+      nr[id - Hq] = block_sum(pr, id - Hq, id - Hq);
+  }
+  __syncthreads();
+  // num[h][h'] becomes sim(h, h') in place
+  for (int id = threadIdx.x; id < Hq * Hq; id += blockDim.x) {
+    const int h = id / Hq, hp = id % Hq;
+    num[id] = block_sum(pn, h, hp) / sqrt(na[h] * nr[hp]);
   }
   __syncthreads();
   for (int id = threadIdx.x; id < Hkv * Hkv; id += blockDim.x) {
     const int ga = id / Hkv, gr = id % Hkv;
     double s = 0.0;
     for (int i = 0; i < g; ++i)
-      for (int j = 0; j < g; ++j) {
-        const int h = ga * g + i, hp = gr * g + j;
-        s += num[h * Hq + hp] / sqrt(na[h] * nr[hp]);
-      }
+      for (int j = 0; j < g; ++j) s += num[(ga * g + i) * Hq + gr * g + j];
     gsim[id] = s / (g * g);
   }
   __syncthreads();
@@ -346,7 +364,7 @@ extern "C" aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_an
   if (e == cudaSuccess) e = launch_gemm(kg, s);
   if (e == cudaSuccess) e = launch_gemm(qg, s);
   if (e == cudaSuccess) {
-    map_kernel<<<1, 256, 0, s>>>(pn, pa, pr, Hq, Hkv, dh, lab, num, na, nr, gsim, map);
+    map_kernel<<<1, 1024, 0, s>>>(pn, pa, pr, Hq, Hkv, dh, lab, num, na, nr, gsim, map);
     e = cudaGetLastError();
   }
   uint32_t h_err = 0;
