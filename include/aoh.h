@@ -188,7 +188,9 @@ aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* 
  *                    group to its most similar anchor group, Eq. sim).
  * Retrieval head i of sequence b attends to the first min(top_k, t + 1)
  * entries of its list; entries outside [0, t] are clamped into it (the
- * reads stay in bounds, the result is then unspecified).
+ * reads stay in bounds, the result is then unspecified). d_head 128 runs on
+ * the tensor cores with the borrowed rows gathered by TMA; d_head 64 on the
+ * CUDA-core kernel.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,

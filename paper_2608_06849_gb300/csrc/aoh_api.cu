@@ -105,6 +105,8 @@ void aoh::record_error(const char* msg) { g_last_error = msg; }
 
 struct aoh_cache {
   CUtensorMap tcr, tcs;  // cache regions for TMA (built once: the buffer does not move)
+  CUtensorMap tcg;       // retrieval rows for row gathers (valid when has_tcg)
+  bool has_tcg = false;
   aoh_config cfg;
   CacheGeom geom;
   std::vector<uint8_t> labels;
@@ -215,6 +217,7 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   h->d_done = h->d_gcounters + n_gcnt;
   h->d_err = h->d_done + 32;
   h->d_partials = reinterpret_cast<float*>(base + 2 * n_lens + n_cnt + n_gcnt + 64);
+  h->has_tcg = make_gather_map(&h->tcg, h->geom, h->kv);
   if (!make_cache_region_maps(&h->tcr, &h->tcs, h->geom, h->kv)) {
     cudaFree(h->meta);
     delete h;
@@ -395,6 +398,7 @@ aoh_status prepare_decode(const void* q, const void* k_new, const void* v_new, a
   }
   a.tcr = cache->tcr;
   a.tcs = cache->tcs;
+  if (cache->has_tcg) a.tcg = cache->tcg;
   a.geom = g;
   a.q = q;
   a.k_new = k_new;
@@ -485,17 +489,21 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
         return fail(AOH_ERR_INVALID, "group_map[%d] = %d is outside [0, %d)", i, group_map[i], n_anchor_groups);
     for (int i = 0; i < g.n_r; ++i) a.idx_map[i] = (uint8_t)group_map[i];
   }
+  a.idx = g.n_r > 0 ? indices : nullptr;
+  a.top_k = top_k;
+  a.n_idx_groups = n_anchor_groups;
+  // d_head 128: the tcgen05 kernel gathers the borrowed rows (tile::gather4),
+  // a gathered row weighing kGatherWeight contiguous rows in the CTA split
+  const bool tc = decode_uses_tc(g.D, g.G) && (g.n_r == 0 || cache->has_tcg);
+  a.gather_w = tc ? kGatherWeight : 1;
   // every retrieval item now holds min(top_k, t + 1) rows
   total = 0;
   for (int b = 0; b < g.B; ++b) {
     const long long t1 = cache->lens[b] + 1;
-    total += g.n_r * std::min<long long>(t1, top_k) + g.n_s * std::min<long long>(t1, g.S + g.W);
+    total += g.n_r * std::min<long long>(t1, top_k) * a.gather_w + g.n_s * std::min<long long>(t1, g.S + g.W);
   }
-  a.idx = g.n_r > 0 ? indices : nullptr;
-  a.top_k = top_k;
-  a.n_idx_groups = n_anchor_groups;
-  a.n_ctas = decode_cc_ctas(total, cache->num_sms);
-  cudaError_t e = launch_decode_cc(a, (cudaStream_t)stream);
+  a.n_ctas = tc ? decode_tc_ctas(total, cache->num_sms) : decode_cc_ctas(total, cache->num_sms);
+  cudaError_t e = tc ? launch_decode_tc(a, (cudaStream_t)stream) : launch_decode_cc(a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "reuse decode kernel launch");
   for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
   return AOH_OK;

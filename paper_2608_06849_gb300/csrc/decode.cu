@@ -2,8 +2,9 @@
 // 5, "Decode Stage", Eq. 8): one new token per sequence; retrieval KV heads
 // attend over their whole history, streaming KV heads over their S sink + W
 // window slots. This kernel serves d_head 64 (d_head 128 runs on the tensor
-// cores, decode_tc.cu), and both sizes in the H2Share reuse step, whose
-// retrieval rows are borrowed positions gathered one row at a time.
+// cores, decode_tc.cu), including the d_head 64 H2Share reuse step, whose
+// retrieval rows are borrowed positions gathered one row at a time (and d_head
+// 128 when the tcgen05 kernel's gather map cannot address the cache).
 //
 // One CTA = one (sequence b, KV head, split) work unit; a split is a
 // contiguous range of cache rows. All G query heads of the GQA group are
@@ -176,9 +177,25 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
             reinterpret_cast<const uint4*>(vn)[lane];
       }
       if (indexed) {
-        // one 1D bulk copy per borrowed row, spread over the warp; indices are
-        // clamped to the rows held, so a bad list cannot read out of bounds
+        // one 1D bulk copy per borrowed row, spread over the warp (lane l
+        // copies rows l, l + 32, ... of a tile); indices are clamped to the
+        // rows held, so a bad list cannot read out of bounds. A tile's
+        // indices are loaded one tile ahead, while the producer waits for a
+        // free stage: read at the tile itself, that load's latency under the
+        // HBM stream would stall every stage.
+        constexpr int RPL = TOK / 32;  // rows per lane and tile
+        static_assert(TOK % 32 == 0, "tile rows");
+        int nxt[RPL];
+#pragma unroll
+        for (int r = 0; r < RPL; ++r) nxt[r] = lo + r * 32 + lane < hi ? __ldg(rowlist + lo + r * 32 + lane) : 0;
         for (int row0 = lo; row0 < hi; row0 += TOK, ++it) {
+          int cur[RPL];
+#pragma unroll
+          for (int r = 0; r < RPL; ++r) {
+            cur[r] = nxt[r];
+            const int j = row0 + TOK + r * 32 + lane;
+            if (j < hi) nxt[r] = __ldg(rowlist + j);
+          }
           const int st = it % NST;
           int ok = 1;
           if (lane == 0) {
@@ -193,10 +210,14 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
           if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)cnt * RB * 2);
           __syncwarp();
           uint8_t* ks = smem + st * C::STAGE_BYTES;
-          for (int r = lane; r < cnt; r += 32) {
-            const int cr = min(max(__ldg(rowlist + row0 + r), 0), t);
-            bulk_g2s(ks + (size_t)r * RB, cr == xr ? kn : Kc + (size_t)cr * RB, RB, &full[st]);
-            bulk_g2s(ks + (size_t)(TOK + r) * RB, cr == xr ? vn : Vc + (size_t)cr * RB, RB, &full[st]);
+#pragma unroll
+          for (int r = 0; r < RPL; ++r) {
+            const int rr = r * 32 + lane;
+            if (rr < cnt) {
+              const int cr = min(max(cur[r], 0), t);
+              bulk_g2s(ks + (size_t)rr * RB, cr == xr ? kn : Kc + (size_t)cr * RB, RB, &full[st]);
+              bulk_g2s(ks + (size_t)(TOK + rr) * RB, cr == xr ? vn : Vc + (size_t)cr * RB, RB, &full[st]);
+            }
           }
           __syncwarp();
         }

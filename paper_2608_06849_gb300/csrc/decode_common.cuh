@@ -39,6 +39,34 @@ __device__ __forceinline__ int item_rows(const DecodeArgs& a, int id, const int*
   return min(t + 1, g.S + g.W);
 }
 
+// Work units of item `id`: its rows, each gathered row of the reuse step
+// weighted by gather_w. The CTAs split the units equally.
+__device__ __forceinline__ int item_weight(const DecodeArgs& a, int id) {
+  return (a.idx != nullptr && id % (a.geom.n_r + a.geom.n_s) < a.geom.n_r) ? a.gather_w : 1;
+}
+__device__ __forceinline__ long long item_units(const DecodeArgs& a, int id, const int* lens_s = nullptr) {
+  return (long long)item_rows(a, id, lens_s) * item_weight(a, id);
+}
+
+// The rows of item `id` (at unit offset off) that the CTA with unit range
+// [start, end) owns: row r sits at unit off + r * w, so every row belongs to
+// exactly one CTA. lo >= hi when the CTA owns none.
+struct Span {
+  int rows, w, lo, hi;
+  long long units;
+};
+__device__ __forceinline__ Span item_span(const DecodeArgs& a, int id, const int* lens_s, long long off,
+                                          long long start, long long end) {
+  Span s;
+  s.rows = item_rows(a, id, lens_s);
+  s.w = item_weight(a, id);
+  s.units = (long long)s.rows * s.w;
+  const long long ulo = max(start, off) - off, uhi = min(end, off + s.units) - off;
+  s.lo = (int)((ulo + s.w - 1) / s.w);
+  s.hi = uhi > ulo ? (int)((uhi + s.w - 1) / s.w) : s.lo;
+  return s;
+}
+
 // CTA whose row range contains global row x.
 __device__ __forceinline__ int cta_of(long long x, long long total, int P) {
   return (int)(((x + 1) * (long long)P - 1) / total);
@@ -59,7 +87,7 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* w
   const int per = (n_items + THREADS - 1) / THREADS;
   const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
   long long mine = 0;
-  for (int id = i0; id < i1; ++id) mine += item_rows(a, id, lens_s);
+  for (int id = i0; id < i1; ++id) mine += item_units(a, id, lens_s);
   long long inc = mine;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -87,7 +115,7 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* w
   if (i0 < i1 && off <= start && start < off + mine) {
     int id = i0;
     while (true) {
-      const int r = item_rows(a, id, lens_s);
+      const long long r = item_units(a, id, lens_s);
       if (start < off + r) break;
       off += r;
       ++id;

@@ -27,7 +27,13 @@
 //              zero weight times a NaN is NaN.
 //   warp 4     TMA producer: K and V tiles of one (sequence, KV head) region
 //              into a 3-stage ring (4D tensor maps over the cache regions,
-//              128-byte swizzle, rows past the region read as zeros).
+//              128-byte swizzle, rows past the region read as zeros). In the
+//              H2Share reuse step a retrieval item's rows are borrowed
+//              positions: the warp's lanes gather them four at a time
+//              (tile::gather4 over a one-row-box map of all retrieval rows),
+//              and the CTAs split the step's rows with each gathered row
+//              weighing kGatherWeight contiguous rows (a row gather costs
+//              more than its share of a streamed tile).
 //   warp 5     TMEM owner and MMA issuer. Loads each item's Q into one of two
 //              swizzled buffers, writes the new token's K/V row over its
 //              (stale) cache row in the landed tile and appends it to the
@@ -67,7 +73,8 @@ constexpr int NBAR = 2 * kNS + 2 + 2 + 2 + 2 + 1 + 1;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
 constexpr int kLensCap = 2048;                // sequence lengths mirrored in shared memory
 constexpr int OFF_LENS = OFF_MISC + 64;
-constexpr int SMEM = OFF_LENS + kLensCap * 4 + 1024;
+constexpr int OFF_PATCH = OFF_LENS + kLensCap * 4;  // [kNS][4] new-token slot masks (gathered tiles)
+constexpr int SMEM = OFF_PATCH + kNS * 16 + 1024;
 constexpr uint32_t IDESC_S = idesc_bf16(kBN, kN, false, false);
 constexpr uint32_t IDESC_PV = idesc_bf16(kD, kN, false, true);
 static_assert(SMEM <= 232448, "shared memory");
@@ -99,6 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   long long* sh64 = reinterpret_cast<long long*>(smem + OFF_MISC + 8);  // [0] total, [1] first offset
   int* sh32 = reinterpret_cast<int*>(sh64 + 2);                         // [0] first item, [1] merge flag
   int* lens_s = reinterpret_cast<int*>(smem + OFF_LENS);
+  uint32_t* patch = reinterpret_cast<uint32_t*>(smem + OFF_PATCH);
 
   const CacheGeom& g = a.geom;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -157,40 +165,100 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
 
   if (warp == 4) {
     // ------------------------------------------------------------ producer
+    // Contiguous items: lane 0 loads 128-row K and V tiles of the region.
+    // Retrieval items of the H2Share reuse step (a.idx): every lane gathers
+    // four of a tile's 128 borrowed rows (tile::gather4 over the gather map,
+    // one instruction per row quad, 64-column half and K or V), with the
+    // tile's indices loaded one tile ahead. Slots past the item's rows read
+    // row 0 (the softmax gives them zero weight); slots holding the new
+    // token (position t, not in the cache yet) read row 0 too and are
+    // listed in the stage's patch mask for the MMA warp to overwrite.
     if (lane == 0) {
-      if (g.n_r > 0) prefetch_tmap(&a.tcr);
+      if (g.n_r > 0) prefetch_tmap(a.idx ? &a.tcg : &a.tcr);
       if (g.n_s > 0) prefetch_tmap(&a.tcs);
-      int it = 0;
-      bool ok = true;
-      long long off = first_off;
-      for (int id = first_id; id < n_items && off < end && ok; ++id) {
-        const int rows = dec::item_rows(a, id, ls);
-        const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
-        off += rows;
-        if (lo >= hi) continue;
-        const int b = id / HK, k = id - b * HK;
-        const bool strm = k >= g.n_r;
-        const int region = strm ? b * g.n_s + (k - g.n_r) : b * g.n_r + k;
-        const CUtensorMap* map = strm ? &a.tcs : &a.tcr;
+    }
+    int it = 0;
+    bool ok = true;
+    long long off = first_off;
+    for (int id = first_id; id < n_items && off < end && ok; ++id) {
+      const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
+      const int rows = sp.rows, lo = sp.lo, hi = sp.hi;
+      off += sp.units;
+      if (lo >= hi) continue;
+      const int b = id / HK, k = id - b * HK;
+      const bool strm = k >= g.n_r;
+      const int region = strm ? b * g.n_s + (k - g.n_r) : b * g.n_r + k;
+      if (a.idx != nullptr && !strm) {
+        const int32_t* rowlist = a.idx + ((size_t)b * a.n_idx_groups + a.idx_map[k]) * a.top_k;
+        const int t = dec::seq_len(a, b, ls);
+        const int kbase = region * 2 * g.max_seq, vbase = kbase + g.max_seq;
+        int nxt[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) nxt[j] = lo + 4 * lane + j < hi ? __ldg(rowlist + lo + 4 * lane + j) : 0;
         for (int row0 = lo; row0 < hi; row0 += kBN) {
+          int cr[4];
+          uint32_t newrow[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const bool valid = row0 + 4 * lane + j < hi;
+            const int c = min(max(nxt[j], 0), t);
+            newrow[j] = __ballot_sync(0xffffffffu, valid && c == t);
+            cr[j] = valid && c != t ? c : 0;
+            const int jn = row0 + kBN + 4 * lane + j;
+            if (jn < hi) nxt[j] = __ldg(rowlist + jn);
+          }
           const int st = it % kNS;
-          if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
+          int go = 1;
+          if (lane == 0) {
+            if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) go = 0;
+            if (go) {
+              // slot 4 * l + j of the tile is bit l of newrow[j]
+#pragma unroll
+              for (int j = 0; j < 4; ++j) patch[st * 4 + j] = newrow[j];
+              mbar_arrive_expect_tx(&full[st], kStage);
+            }
+          }
+          if (!__shfl_sync(0xffffffffu, go, 0)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&full[st], kStage);
-          uint8_t* dst = sKV + st * kStage;
+          uint8_t* dst = sKV + st * kStage + 4 * lane * 128;
 #pragma unroll
-          for (int sel = 0; sel < 2; ++sel)
-#pragma unroll
-            for (int db = 0; db < 2; ++db)
-              tma_load_4d(dst + sel * kTile + db * kBox, map, db * 64, row0, sel, region, &full[st]);
+          for (int db = 0; db < 2; ++db) {
+            tma_gather4(dst + db * kBox, &a.tcg, db * 64, kbase + cr[0], kbase + cr[1], kbase + cr[2],
+                        kbase + cr[3], &full[st]);
+            tma_gather4(dst + kTile + db * kBox, &a.tcg, db * 64, vbase + cr[0], vbase + cr[1], vbase + cr[2],
+                        vbase + cr[3], &full[st]);
+          }
           ++it;
         }
+      } else {
+        if (lane == 0) {
+          const CUtensorMap* map = strm ? &a.tcs : &a.tcr;
+          for (int row0 = lo; row0 < hi; row0 += kBN) {
+            const int st = it % kNS;
+            if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[st], kStage);
+            uint8_t* dst = sKV + st * kStage;
+#pragma unroll
+            for (int sel = 0; sel < 2; ++sel)
+#pragma unroll
+              for (int db = 0; db < 2; ++db)
+                tma_load_4d(dst + sel * kTile + db * kBox, map, db * 64, row0, sel, region, &full[st]);
+            ++it;
+          }
+        }
+        // lane 0 alone advanced the ring counter and saw the waits
+        it = __shfl_sync(0xffffffffu, it, 0);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       }
-      // every issued copy lands before the CTA can exit
-      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) wait_bar(&full[j % kNS], (j / kNS) & 1, a.err, abort_flag);
     }
+    // every issued copy lands before the CTA can exit
+    if (lane == 0)
+      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) wait_bar(&full[j % kNS], (j / kNS) & 1, a.err, abort_flag);
   } else if (warp == 5) {
     // ------------------------------------------------------------ MMA issuer
     const uint32_t kv_addr = smem_u32(sKV), q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
@@ -257,13 +325,17 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       const size_t new_off = ((size_t)b * g.Hkv + kvh) * kD + ch * 8;
       nvr = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(lane < 16 ? a.k_new : a.v_new) + new_off);
     };
-    if (first_id < n_items) fetch_inputs(first_id);
+    int fetched = -1;  // the item whose inputs the registers hold
+    if (first_id < n_items) {
+      fetch_inputs(first_id);
+      fetched = first_id;
+    }
 
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
-      const int rows = dec::item_rows(a, id, ls);
-      const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
-      off += rows;
+      const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
+      const int rows = sp.rows, lo = sp.lo, hi = sp.hi;
+      off += sp.units;
       if (lo >= hi) continue;
       const int b = id / HK, k = id - b * HK;
       const bool strm = k >= g.n_r;
@@ -277,6 +349,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       // this item's Q into buffer item_k & 1, last read by the MMAs of item item_k - 2
       wait_ofree(item_k - 1);
       if (!ok) break;
+      if (fetched != id) {  // an item skipped by this CTA took the prefetch
+        fetch_inputs(id);
+        fetched = id;
+      }
       {
         uint8_t* qs = sQ + (item_k & 1) * kOpBuf;
 #pragma unroll
@@ -292,18 +368,43 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       }
       const uint4 nv = nvr;
       // the next item of this CTA's range starts at its row 0
-      if (off < end && id + 1 < n_items) fetch_inputs(id + 1);
+      if (off < end && id + 1 < n_items) {
+        fetch_inputs(id + 1);
+        fetched = id + 1;
+      }
 
+      // H2Share reuse step: this retrieval item's rows are gathered
+      const bool gathered = a.idx != nullptr && !strm;
       for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
         const int st = it % kNS;
         const int cnt = min(kBN, hi - row0);
         wait_warp(&full[st], (it / kNS) & 1);
         if (!ok) break;
-        if (xr >= row0 && xr < row0 + cnt) {
-          const int r = xr - row0;
+        auto put_new_row = [&](int r) {  // the new token's K / V chunk into tile slot r
           uint8_t* dst = sKV + st * kStage + (lane < 16 ? 0 : kTile) + (ch >> 3) * kBox + r * 128 +
                          (((ch & 7) ^ (r & 7)) << 4);
           *reinterpret_cast<uint4*>(dst) = nv;
+        };
+        if (gathered) {
+          // slots that borrow position t; the item's owner of row 0 appends it
+          bool any = false;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            uint32_t m = patch[st * 4 + j];
+            any = any || m != 0u;
+            while (m) {
+              const int l = __ffs(m) - 1;
+              m &= m - 1;
+              put_new_row(4 * l + j);
+            }
+          }
+          if (row0 == 0) *reinterpret_cast<uint4*>((lane < 16 ? Kc : Vc) + (size_t)xr * kD + ch * 8) = nv;
+          if (any) {
+            fence_proxy_async_smem();
+            __syncwarp();
+          }
+        } else if (xr >= row0 && xr < row0 + cnt) {
+          put_new_row(xr - row0);
           *reinterpret_cast<uint4*>((lane < 16 ? Kc : Vc) + (size_t)xr * kD + ch * 8) = nv;  // append
           fence_proxy_async_smem();
           __syncwarp();
@@ -354,10 +455,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
     bool ok = true, local_ok = true;
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
-      const int rows = dec::item_rows(a, id, ls);
+      const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
+      const int rows = sp.rows, lo = sp.lo, hi = sp.hi;
       const long long item_off = off;
-      const int lo = (int)(max(start, off) - off), hi = (int)(min(end, off + rows) - off);
-      off += rows;
+      off += sp.units;
       if (lo >= hi) continue;
       const int b = id / HK, k = id - b * HK;
       const bool strm = k >= g.n_r;
@@ -482,7 +583,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
 #pragma unroll
       for (int h = 0; h < G; ++h) L[h] = (lsum[h] + lsum[16 + h]) + (lsum[32 + h] + lsum[48 + h]);
 
-      const int f = dec::cta_of(item_off, total, P), lst = dec::cta_of(item_off + rows - 1, total, P);
+      const int f = dec::cta_of(item_off, total, P);
+      const int lst = dec::cta_of(item_off + (long long)(rows - 1) * sp.w, total, P);
       bf16* outp = static_cast<bf16*>(a.out) + ((size_t)b * g.Hq + (size_t)kvh * G) * kD;
       float2* st = (a.scores != nullptr && !strm) ? a.score_stats + (size_t)(b * g.n_r + k) * G : nullptr;
       if (f == lst) {
@@ -550,6 +652,22 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
 }  // namespace
 
 bool decode_uses_tc(int D, int G) { return D == kD && ((G >= 1 && G <= 8) || G == 16); }
+
+bool make_gather_map(CUtensorMap* tcg, const CacheGeom& g, const void* kv) {
+  if (g.D != kD || g.n_r <= 0) return false;
+  const long long rows = (long long)g.B * g.n_r * 2 * g.max_seq;
+  if (rows >= (1LL << 31)) return false;  // row coordinates are 32-bit
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+  cuuint32_t box[2] = {64, 1};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(tcg, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+            const_cast<bf16*>(static_cast<const bf16*>(kv) + g.r_region(0, 0)), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 // One CTA per SM; small steps use fewer, at least 512 rows each.
 int decode_tc_ctas(long long total_rows, int num_sms) {

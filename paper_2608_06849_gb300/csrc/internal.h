@@ -45,6 +45,8 @@ struct CacheGeom {
 
 struct DecodeArgs {
   CUtensorMap tcr, tcs;  // cache regions (see PrefillTcArgs); read by the tcgen05 kernel
+  CUtensorMap tcg;       // retrieval rows as one [B * n_r * 2 * max_seq][D] matrix, one-row
+                         // box (row gathers of the H2Share reuse step on the tcgen05 kernel)
   CacheGeom geom;
   const void* q;      // [B][Hq][D]
   const void* k_new;  // [B][Hkv][D]
@@ -67,12 +69,15 @@ struct DecodeArgs {
   float* scores = nullptr;
   int score_stride = 0;
   float2* score_stats = nullptr;
-  // H2Share reuse step (CUDA-core kernel): when non-null, retrieval item
+  // H2Share reuse step (both decode kernels): when non-null, retrieval item
   // (b, i) attends only to the cache rows idx[(b * n_idx_groups + idx_map[i]) *
   // top_k + r], r < min(top_k, t + 1).
   const int32_t* idx = nullptr;
   int top_k = 0;
   int n_idx_groups = 0;
+  // Work units per gathered row when the CTAs split the step (a borrowed row
+  // costs several contiguous rows); 1 everywhere else.
+  int gather_w = 1;
   uint8_t idx_map[kMaxKvHeads] = {};
 };
 
@@ -120,6 +125,9 @@ bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv);
 // [regions][K, V][capacity rows][D] with box [1][1][128][64] and 128-byte
 // swizzle; a kind with no heads leaves its map untouched.
 bool make_cache_region_maps(CUtensorMap* tcr, CUtensorMap* tcs, const CacheGeom& g, const void* kv);
+// The gather map of DecodeArgs::tcg (d_head 128, retrieval heads present,
+// fewer than 2^31 retrieval rows); false if it cannot be built.
+bool make_gather_map(CUtensorMap* tcg, const CacheGeom& g, const void* kv);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
 // The CUDA-core decode kernel for any supported (D, G) (the H2Share reuse
@@ -143,6 +151,10 @@ cudaError_t launch_h2_topk(float* ws, int max_seq, const int32_t* lens, int B, i
 int decode_ctas(long long total_rows, int num_sms, int D, int G);
 // The tcgen05 decode kernel serves (D, G) (else the CUDA-core kernel does).
 bool decode_uses_tc(int D, int G);
+// Work units of one gathered row in the reuse step's split on the tcgen05
+// kernel (a 256-byte row gather against a contiguous row's share of a tile
+// stream; measured).
+constexpr int kGatherWeight = 4;
 int decode_tc_ctas(long long total_rows, int num_sms);
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
