@@ -182,7 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
       const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
-      const int rows = sp.rows, lo = sp.lo, hi = sp.hi;
+      const int lo = sp.lo, hi = sp.hi;
       off += sp.units;
       if (lo >= hi) continue;
       const int b = id / HK, k = id - b * HK;
@@ -334,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
       const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
-      const int rows = sp.rows, lo = sp.lo, hi = sp.hi;
+      const int lo = sp.lo, hi = sp.hi;
       off += sp.units;
       if (lo >= hi) continue;
       const int b = id / HK, k = id - b * HK;

@@ -133,11 +133,13 @@ __global__ void __launch_bounds__(kSelThreads) h2_select_kernel(const int32_t* l
   const int n = __ldcg(&lens[b]);
   const float* imp = imp_all + (size_t)item * stride;
   int32_t* out = idx_all + (size_t)item * top_k;
+  uint32_t* hist = hist_all + (size_t)item * kBins;
   if (n <= top_k) {
     for (int j = threadIdx.x; j < top_k; j += kSelThreads) out[j] = j < n ? j : -1;
+    // the importance kernel counted this step's rows: zero them for the next
+    for (int i = threadIdx.x; i < kBins; i += kSelThreads) hist[i] = 0u;
     return;
   }
-  uint32_t* hist = hist_all + (size_t)item * kBins;
   for (int i = threadIdx.x; i < kBins; i += kSelThreads) {
     h2[i] = __ldcg(hist + i);
     hist[i] = 0u;  // zero again for the next step
@@ -254,10 +256,14 @@ __global__ void __launch_bounds__(kSelThreads) h2_select_kernel(const int32_t* l
 
 }  // namespace
 
+// Every segment starts on a 16-byte boundary (the head states are float2,
+// and max_seq may be odd).
+inline size_t pad4(size_t n) { return (n + 3) / 4 * 4; }
+
 size_t h2_workspace_floats(int B, int n_r, int G, int max_seq) {
   const size_t items = (size_t)B * n_r;
   // scores, importance, per-head (max, sum) states (float2), histograms (uint32)
-  return items * (size_t)max_seq * (G + 1) + items * G * 2 + items * kBins;
+  return pad4(items * (size_t)max_seq * G) + pad4(items * (size_t)max_seq) + pad4(items * G * 2) + items * kBins;
 }
 
 namespace {
@@ -271,9 +277,9 @@ H2Layout h2_layout(float* ws, int B, int n_r, int G, int max_seq) {
   const size_t items = (size_t)B * n_r;
   H2Layout l;
   l.scores = ws;
-  l.imp = l.scores + items * (size_t)max_seq * G;
-  l.stats = reinterpret_cast<float2*>(l.imp + items * (size_t)max_seq);
-  l.hist = reinterpret_cast<uint32_t*>(reinterpret_cast<float*>(l.stats) + items * G * 2);
+  l.imp = l.scores + pad4(items * (size_t)max_seq * G);
+  l.stats = reinterpret_cast<float2*>(l.imp + pad4(items * (size_t)max_seq));
+  l.hist = reinterpret_cast<uint32_t*>(reinterpret_cast<float*>(l.stats) + pad4(items * G * 2));
   return l;
 }
 }  // namespace

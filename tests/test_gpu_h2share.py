@@ -87,6 +87,57 @@ def test_anchor_step_selects_top_k(B, Hq, Hkv, T, labels, top_k):
     cache.close()
 
 
+def test_anchor_selection_when_length_crosses_top_k():
+    """Steps with t + 1 <= top_k keep every row; the first step beyond it
+    must rank from that step's importances alone."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, top_k, steps = 2, 8, 2, 128, 60, 4, 16, 62, 4
+    labels = [0, 1]
+    g = Hq // Hkv
+    cache, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, steps, 81)
+    wl = Workload("cross", B, Hq, Hkv, D, T, steps, S, W, 1, seed=9)
+    kall = [f64(k[b]) for b in range(B)]
+    for step in range(steps):
+        dq, dk, dv = decode_inputs(wl, step, device="cuda")
+        idx = torch.full((B, 1, top_k), -7, dtype=torch.int32, device="cuda")
+        cache.decode_step_anchor(dq, dk, dv, torch.empty_like(dq), top_k, idx)
+        torch.cuda.synchronize()
+        sel = idx.cpu().numpy()
+        for b in range(B):
+            kall[b] = np.concatenate([kall[b], f64(dk[b])[None]])
+            imp = ohs.group_importance(f64(dq[b])[:g], kall[b][:, 0])
+            _check_selection(sel[b, 0], imp, top_k)
+    cache.close()
+
+
+def test_anchor_selection_with_one_crowded_bucket():
+    """Identical keys give every cached position the same importance (the
+    new token's differs): one histogram bucket holds more rows than the
+    candidate list, so the threshold comes from full passes, and the tied
+    rows are taken in position order across several chunks."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, top_k = 1, 8, 2, 128, 20000, 4, 64, 9000
+    labels = [0, 1]
+    g = Hq // Hkv
+    cache = aoh.Cache(B, Hq, Hkv, D, T + 1, S, W, labels)
+    k = randn_bf16((B, 1, Hkv, D), 91, "cuda").expand(B, T, Hkv, D).contiguous()
+    v = randn_bf16((B, T, Hkv, D), 92, "cuda")
+    cache.prefill(None, k, v, None)
+    wl = Workload("crowd", B, Hq, Hkv, D, T, 1, S, W, 1, seed=10)
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    idx = torch.full((B, 1, top_k), -7, dtype=torch.int32, device="cuda")
+    cache.decode_step_anchor(dq, dk, dv, torch.empty_like(dq), top_k, idx)
+    torch.cuda.synchronize()
+    sel = idx.cpu().numpy()[0, 0]
+    kk = np.concatenate([f64(k[0]), f64(dk[0])[None]])
+    imp = ohs.group_importance(f64(dq[0])[:g], kk[:, 0])
+    _check_selection(sel, imp, top_k)
+    # the tied positions are taken lowest first
+    tied = sel[sel < T]
+    assert np.array_equal(tied[: len(tied)], np.arange(len(tied))) or imp[T] < imp[0]
+    cache.close()
+
+
 def _reuse_case(B, Hq, Hkv, D, T, S, W, labels, top_k, n_anchor, group_map, steps=2, seed=41):
     ensure_lib()
     g = Hq // Hkv
