@@ -55,7 +55,8 @@ struct Problem {
   CUtensorMap ta, tb;  // A [M][K], B [N][K], bf16, row-major
   float* c;            // store mode: C [M][N] fp32
   const float* r;      // trace mode: key-side matrix, leading dimension ldr
-  double* part;        // trace mode: [M/32][N/32] block partials
+  double* out;         // trace mode: per head pair tr(A B), out[h * (N / d_head) + h']
+  int out_diag;        // trace mode: only pairs h == h', to out[h]
   int M, N, ldr;
   int diag;            // only tiles (t, t)
   int tiles;           // CTAs of this problem
@@ -107,6 +108,7 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  __shared__ double red[4][4];  // trace mode: [row quarter][column chunk] partials of the tile
   // the next launch on the stream (the query side after the key side) may
   // start its main loop now; it waits for this grid only before its epilogue
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -151,7 +153,11 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
     const bool ok = __all_sync(0xffffffffu, wait_bar(done, 0, a.err, abort_flag));
     const int row0 = tm * kTM + q4 * 32;
     // trace mode reads the key-side matrices of the previous launch
-    if (a.trace) asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (a.trace) {
+      asm volatile("griddepcontrol.wait;" ::: "memory");
+      if (lane < 4) red[q4][lane] = 0.0;
+      __syncwarp();
+    }
     if (ok && row0 < P.M) {
       tc_fence_after();
       const int r = row0 + lane;
@@ -176,7 +182,7 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
           double acc = ((double)s[0] + (double)s[1]) + ((double)s[2] + (double)s[3]);
 #pragma unroll
           for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-          if (lane == 0) P.part[(size_t)(row0 / 32) * (P.N / 32) + col0 / 32] = acc;
+          if (lane == 0) red[q4][c] = acc;
         } else {
           float* dst = P.c + (size_t)r * P.N + col0;
 #pragma unroll
@@ -184,6 +190,23 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
             *reinterpret_cast<float4*>(dst + e) = make_float4(__uint_as_float(v[e]), __uint_as_float(v[e + 1]),
                                                               __uint_as_float(v[e + 2]), __uint_as_float(v[e + 3]));
         }
+      }
+    }
+    if (a.trace) {
+      // the tile holds whole head pairs (128 / d_head heads a side); each
+      // pair's trace is the sum of its 32 x 32 blocks, rows then columns
+      named_barrier_sync(1, 128);
+      if (threadIdx.x == 64) {
+        const int R = kTM / a.dh, W = a.dh / 32, Hr = P.M / a.dh, Hc = P.N / a.dh;
+        for (int ha = 0; ha < R; ++ha)
+          for (int hb = 0; hb < R; ++hb) {
+            const int h = tm * R + ha, hp = tn * R + hb;
+            if (h >= Hr || hp >= Hc || (P.out_diag && h != hp)) continue;
+            double sum = 0.0;
+            for (int x = 0; x < W; ++x)
+              for (int y = 0; y < W; ++y) sum += red[ha * W + x][hb * W + y];
+            P.out[P.out_diag ? h : (size_t)h * Hc + hp] = sum;
+          }
       }
     }
   }
@@ -208,12 +231,13 @@ bool make_2d_map(CUtensorMap* map, const void* base, int rows, int K) {
 
 // One problem of a launch: C = A B^T with A [M][K], B [N][K].
 bool add_problem(GemmArgs& g, const void* A, int M, const void* B, int N, int K, bool diag, float* c,
-                 const float* r, int ldr, double* part) {
+                 const float* r, int ldr, double* out) {
   Problem& p = g.p[g.n_problems++];
   if (!make_2d_map(&p.ta, A, M, K) || !make_2d_map(&p.tb, B, N, K)) return false;
   p.c = c;
   p.r = r;
-  p.part = part;
+  p.out = out;
+  p.out_diag = diag ? 1 : 0;
   p.M = M;
   p.N = N;
   p.ldr = ldr;
@@ -251,38 +275,21 @@ struct Labels {
   uint8_t a[kMaxKvHeads], r[kMaxKvHeads];
 };
 
-// Head-pair traces from the block partials (each a sum over its (d_head/32)^2
-// blocks in a fixed order), then the group means and the argmax. parts:
-// pn [Hq d_head / 32]^2 for the numerators, pa / pr the same shape with only
-// the diagonal head blocks used. fp64 divides and square roots are slow on
-// this part, so each phase spreads its items over the block's threads.
-__global__ void map_kernel(const double* pn, const double* pa, const double* pr, int Hq, int Hkv, int dh,
-                           Labels lab, double* num, double* na, double* nr, double* gsim, int32_t* map) {
-  const int nb = dh / 32, ld = Hq * nb, g = Hq / Hkv;
-  auto block_sum = [&](const double* p, int h, int hp) {
-    double s = 0.0;
-    for (int x = 0; x < nb; ++x)
-      for (int y = 0; y < nb; ++y) s += p[(size_t)(h * nb + x) * ld + hp * nb + y];
-    return s;
-  };
-  for (int id = threadIdx.x; id < 2 * Hq; id += blockDim.x) {
-    if (id < Hq)
-      na[id] = block_sum(pa, id, id);
-    else
-      nr[id - Hq] = block_sum(pr, id - Hq, id - Hq);
-  }
+// sim(h, h') = tr(A B) / sqrt(n_a(h) n_r(h')) from the traces, then the
+// group means and the argmax. fp64 divides and square roots are slow on this
+// part: 2 Hq of them (the inverse norms), spread over the block's threads.
+__global__ void map_kernel(const double* num, const double* na, const double* nr, int Hq, int Hkv, Labels lab,
+                           double* inv, double* sim, double* gsim, int32_t* map) {
+  const int g = Hq / Hkv;
+  for (int id = threadIdx.x; id < 2 * Hq; id += blockDim.x) inv[id] = 1.0 / sqrt(id < Hq ? na[id] : nr[id - Hq]);
   __syncthreads();
-  // num[h][h'] becomes sim(h, h') in place
-  for (int id = threadIdx.x; id < Hq * Hq; id += blockDim.x) {
-    const int h = id / Hq, hp = id % Hq;
-    num[id] = block_sum(pn, h, hp) / sqrt(na[h] * nr[hp]);
-  }
+  for (int id = threadIdx.x; id < Hq * Hq; id += blockDim.x) sim[id] = num[id] * inv[id / Hq] * inv[Hq + id % Hq];
   __syncthreads();
   for (int id = threadIdx.x; id < Hkv * Hkv; id += blockDim.x) {
     const int ga = id / Hkv, gr = id % Hkv;
     double s = 0.0;
     for (int i = 0; i < g; ++i)
-      for (int j = 0; j < g; ++j) s += num[(ga * g + i) * Hq + gr * g + j];
+      for (int j = 0; j < g; ++j) s += sim[(ga * g + i) * Hq + gr * g + j];
     gsim[id] = s / (g * g);
   }
   __syncthreads();
@@ -327,23 +334,22 @@ extern "C" aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_an
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int Hq = n_q_heads, Hkv = n_kv_heads, dh = d_head, dm = d_model;
   const int nq = Hq * dh, nk = Hkv * dh;
-  const size_t nparts = (size_t)(nq / 32) * (nq / 32);
-  // key-side Y, G_ka, G_kr; three partial grids; traces; outputs
-  const size_t bytes = 3 * (size_t)nk * nk * 4 + 3 * nparts * 8 + ((size_t)Hq * Hq + 2 * Hq + (size_t)Hkv * Hkv) * 8 +
-                       Hkv * 4 + 256;
+  // key-side Y, G_ka, G_kr; traces (pairs, two norm sets); inverse norms;
+  // head and group similarities; map; error word
+  const size_t bytes = 3 * (size_t)nk * nk * 4 + ((size_t)Hq * Hq + 2 * Hq) * 8 + 2 * (size_t)Hq * 8 +
+                       (size_t)Hq * Hq * 8 + (size_t)Hkv * Hkv * 8 + Hkv * 4 + 256;
   void* ws = nullptr;
   cudaError_t e = cudaMallocAsync(&ws, bytes, s);
   if (e != cudaSuccess) return fail(AOH_ERR_CUDA, "aoh_h2share_map: cudaMallocAsync failed");
   float* Y = static_cast<float*>(ws);
   float* gka = Y + (size_t)nk * nk;
   float* gkr = gka + (size_t)nk * nk;
-  double* pn = reinterpret_cast<double*>(gkr + (size_t)nk * nk);
-  double* pa = pn + nparts;
-  double* pr = pa + nparts;
-  double* num = pr + nparts;
+  double* num = reinterpret_cast<double*>(gkr + (size_t)nk * nk);
   double* na = num + (size_t)Hq * Hq;
   double* nr = na + Hq;
-  double* gsim = nr + Hq;
+  double* inv = nr + Hq;
+  double* sim = inv + 2 * (size_t)Hq;
+  double* gsim = sim + (size_t)Hq * Hq;
   int32_t* map = reinterpret_cast<int32_t*>(gsim + (size_t)Hkv * Hkv);
   uint32_t* err = reinterpret_cast<uint32_t*>(map + Hkv);
   GemmArgs kg{}, qg{};
@@ -356,15 +362,15 @@ extern "C" aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_an
   bool maps_ok = add_problem(kg, w_k_reuse, nk, w_k_anchor, nk, dm, false, Y, nullptr, 0, nullptr) &&
                  add_problem(kg, w_k_anchor, nk, w_k_anchor, nk, dm, false, gka, nullptr, 0, nullptr) &&
                  add_problem(kg, w_k_reuse, nk, w_k_reuse, nk, dm, false, gkr, nullptr, 0, nullptr) &&
-                 add_problem(qg, w_q_anchor, nq, w_q_reuse, nq, dm, false, nullptr, Y, nk, pn) &&
-                 add_problem(qg, w_q_anchor, nq, w_q_anchor, nq, dm, true, nullptr, gka, nk, pa) &&
-                 add_problem(qg, w_q_reuse, nq, w_q_reuse, nq, dm, true, nullptr, gkr, nk, pr);
+                 add_problem(qg, w_q_anchor, nq, w_q_reuse, nq, dm, false, nullptr, Y, nk, num) &&
+                 add_problem(qg, w_q_anchor, nq, w_q_anchor, nq, dm, true, nullptr, gka, nk, na) &&
+                 add_problem(qg, w_q_reuse, nq, w_q_reuse, nq, dm, true, nullptr, gkr, nk, nr);
   if (!maps_ok) e = cudaErrorInvalidValue;
   if (e == cudaSuccess) e = cudaMemsetAsync(err, 0, 4, s);
   if (e == cudaSuccess) e = launch_gemm(kg, s);
   if (e == cudaSuccess) e = launch_gemm(qg, s);
   if (e == cudaSuccess) {
-    map_kernel<<<1, 1024, 0, s>>>(pn, pa, pr, Hq, Hkv, dh, lab, num, na, nr, gsim, map);
+    map_kernel<<<1, 1024, 0, s>>>(num, na, nr, Hq, Hkv, lab, inv, sim, gsim, map);
     e = cudaGetLastError();
   }
   uint32_t h_err = 0;

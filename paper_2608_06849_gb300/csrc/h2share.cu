@@ -38,8 +38,9 @@ constexpr int kSelThreads = 1024;
 constexpr int kBins = 2048;           // top 11 bits
 constexpr int kCand = 8192;           // candidates kept in shared memory
 
+template <int G>
 __global__ void __launch_bounds__(kChunkThreads) h2_imp_kernel(const float* scores, int stride, const int32_t* lens,
-                                                               int n_r, int G, const float2* stats, float* imp_all,
+                                                               int n_r, const float2* stats, float* imp_all,
                                                                uint32_t* hist) {
   __shared__ float Mh[16], Linv[16];
   __shared__ uint32_t sh_hist[kBins];
@@ -54,15 +55,30 @@ __global__ void __launch_bounds__(kChunkThreads) h2_imp_kernel(const float* scor
   __syncthreads();
   const int j0 = chunk * kChunk, j1 = min(n, j0 + kChunk);
   float* imp = imp_all + (size_t)item * stride;
-  for (int j = j0 + threadIdx.x; j < j1; j += kChunkThreads) {
-    float v = 0.f;
-    for (int h = 0; h < G; ++h)
-      v += fast_exp2(__ldcg(scores + ((size_t)item * G + h) * stride + j) - Mh[h]) * Linv[h];
-    imp[j] = v;
-    // warp-aggregated: most importances are tiny and share a few bins
-    const uint32_t bin = __float_as_uint(v) >> 21;
-    const unsigned peers = __match_any_sync(__activemask(), bin);
-    if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&sh_hist[bin], (uint32_t)__popc(peers));
+  // U rows per thread and step, every score load of the step issued before
+  // any is used (the histogram atomics would otherwise keep the next row's
+  // loads from being hoisted, leaving G loads in flight per thread)
+  constexpr int U = 4;
+  for (int jb = j0; jb < j1; jb += U * kChunkThreads) {
+    float sv[U][G];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int j = jb + u * kChunkThreads + threadIdx.x;
+#pragma unroll
+      for (int h = 0; h < G; ++h) sv[u][h] = j < j1 ? __ldcg(scores + ((size_t)item * G + h) * stride + j) : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int j = jb + u * kChunkThreads + threadIdx.x;
+      float v = 0.f;
+#pragma unroll
+      for (int h = 0; h < G; ++h) v += fast_exp2(sv[u][h] - Mh[h]) * Linv[h];
+      if (j < j1) imp[j] = v;
+      // warp-aggregated: most importances are tiny and share a few bins
+      const uint32_t bin = j < j1 ? __float_as_uint(v) >> 21 : 0xffffffffu;
+      const unsigned peers = __match_any_sync(0xffffffffu, bin);
+      if (j < j1 && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&sh_hist[bin], (uint32_t)__popc(peers));
+    }
   }
   __syncthreads();
   for (int i = threadIdx.x; i < kBins; i += kChunkThreads)
@@ -302,7 +318,16 @@ cudaError_t launch_h2_topk(float* ws, int max_seq, const int32_t* lens, int B, i
   const H2Layout l = h2_layout(ws, B, n_r, G, max_seq);
   const size_t items = (size_t)B * n_r;
   const dim3 grid((max_seq + kChunk - 1) / kChunk, (unsigned)items);
-  h2_imp_kernel<<<grid, kChunkThreads, 0, s>>>(l.scores, max_seq, lens, n_r, G, l.stats, l.imp, l.hist);
+  switch (G) {
+#define AOH_IMP(g)                                                                                      \
+  case g:                                                                                               \
+    h2_imp_kernel<g><<<grid, kChunkThreads, 0, s>>>(l.scores, max_seq, lens, n_r, l.stats, l.imp, l.hist); \
+    break;
+    AOH_IMP(1) AOH_IMP(2) AOH_IMP(3) AOH_IMP(4) AOH_IMP(5) AOH_IMP(6) AOH_IMP(7) AOH_IMP(8) AOH_IMP(16)
+#undef AOH_IMP
+    default:
+      return cudaErrorInvalidValue;
+  }
   h2_select_kernel<<<(unsigned)items, kSelThreads, 0, s>>>(lens, n_r, max_seq, top_k, l.imp, l.hist, idx_out);
   return cudaGetLastError();
 }
