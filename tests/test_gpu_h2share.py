@@ -203,6 +203,64 @@ def test_reuse_step_attends_to_borrowed_rows(D, Hq, Hkv, labels, top_k, n_anchor
     _reuse_case(2, Hq, Hkv, D, 900, 4, 50, labels, top_k, n_anchor, gmap)
 
 
+@pytest.mark.parametrize("D,Hq,Hkv,labels", [
+    (128, 8, 2, [0, 1]),       # tensor-core kernel, gathered rows
+    (128, 14, 2, [0, 0]),
+    (64, 8, 2, [1, 0]),        # CUDA-core kernel
+])
+def test_reuse_step_ragged_lengths(D, Hq, Hkv, labels):
+    """Sequences of different lengths, so items of different sizes share the
+    CTAs' weighted split; one list holds the new token, one sequence holds
+    fewer rows than top_k."""
+    ensure_lib()
+    B, S, W, top_k = 3, 4, 40, 200
+    lens = [300, 1100, 37]
+    T = max(lens)
+    g = Hq // Hkv
+    retr = [h for h in range(Hkv) if labels[h] == 0]
+    n_anchor = len(retr)
+    cache = aoh.Cache(B, Hq, Hkv, D, T + 2, S, W, labels)
+    k = randn_bf16((B, T, Hkv, D), 201, "cuda")
+    v = randn_bf16((B, T, Hkv, D), 202, "cuda")
+    cache.prefill(None, k, v, None, seq_lens=lens)
+    wl = Workload("ragged-reuse", B, Hq, Hkv, D, T, 1, S, W, sum(labels), seed=12)
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    rng = np.random.default_rng(5)
+    lists = np.full((B, n_anchor, top_k), -1, dtype=np.int32)
+    for b in range(B):
+        t = lens[b]
+        for a in range(n_anchor):
+            m = min(top_k, t + 1)
+            pick = np.sort(rng.choice(t + 1, size=m, replace=False))
+            if b == 1 and a == 0 and t not in pick:
+                pick[-1] = t               # the new token among the borrowed rows
+            lists[b, a, :m] = np.sort(pick)
+    out = torch.full_like(dq, float("nan"))
+    gmap = list(range(n_anchor))[::-1]
+    cache.decode_step_reuse(dq, dk, dv, out, torch.from_numpy(lists).cuda(), top_k, gmap)
+    torch.cuda.synchronize()
+    for b in range(B):
+        t = lens[b]
+        kk = np.concatenate([f64(k[b, :t]), f64(dk[b])[None]])
+        vv = np.concatenate([f64(v[b, :t]), f64(dv[b])[None]])
+        q = f64(dq[b])
+        full = oatt.decode_step(q, kk, vv, labels, S, W)
+        fmag = oatt.decode_step(q, kk, np.abs(vv), labels, S, W)
+        for kvh in range(Hkv):
+            hs = slice(kvh * g, (kvh + 1) * g)
+            if labels[kvh] == 0:
+                pos = lists[b, gmap[retr.index(kvh)]]
+                pos = pos[pos >= 0]
+                want = ohs.sparse_attend(q[hs], kk[:, kvh], vv[:, kvh], pos)
+                mag = ohs.sparse_attend(q[hs], kk[:, kvh], np.abs(vv[:, kvh]), pos)
+            else:
+                want, mag = full[hs], fmag[hs]
+            assert_matches(f64(out[b, hs]), want, f"ragged reuse b={b} kv={kvh}", mag)
+    assert cache.lens() == [x + 1 for x in lens]
+    cache.check()
+    cache.close()
+
+
 def test_anchor_then_reuse():
     """An anchor layer and a reuse layer of one block at the same step: the
     reuse layer attends to its own K/V at the positions the anchor chose."""
