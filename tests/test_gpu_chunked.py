@@ -78,6 +78,9 @@ CASES = {
     "single_token_chunks": (1, 8, 2, 128, [[40]] + [[1]] * 5, 3, 17, [1, 0]),
     "group7_d128": (1, 14, 2, 128, [[257], [300]], 8, 130, [0, 1]),
     "d64": (1, 8, 2, 64, [[200], [333]], 16, 128, [1, 0]),
+    # 24 sequences: the second chunk's 192 retrieval items, each reading its
+    # sequence's 1024-token prefix, outnumber the SMs
+    "many_sequences": (24, 8, 2, 128, [[1024] * 24, [512] * 24], 4, 64, [0, 1]),
     "ragged_two_seqs": (2, 8, 2, 128, [[300, 77], [100, 400], [260, 5]], 16, 128, [1, 0]),
     "window_equals_chunk": (1, 8, 2, 128, [[256], [256], [256]], 0, 256, [1, 1]),
 }
