@@ -477,7 +477,11 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
   const aoh_status st = prepare_decode(q, k_new, v_new, cache, out, a, total);
   if (st != AOH_OK) return st;
   const CacheGeom& g = cache->geom;
-  if (!decode_cc_supported(g.D, g.G)) return fail(AOH_ERR_UNSUPPORTED, "group size not compiled for the reuse step");
+  // d_head 128: the tcgen05 kernel gathers the borrowed rows (tile::gather4),
+  // a gathered row weighing kGatherWeight contiguous rows in the CTA split
+  const bool tc = decode_uses_tc(g.D, g.G) && (g.n_r == 0 || cache->has_tcg);
+  if (!tc && !decode_cc_supported(g.D, g.G))
+    return fail(AOH_ERR_UNSUPPORTED, "group size not compiled for the reuse step");
   if (top_k < 1) return fail(AOH_ERR_INVALID, "top_k must be >= 1");
   if (g.n_r > 0) {
     if (!indices || !group_map) return fail(AOH_ERR_INVALID, "indices and group_map must not be NULL");
@@ -492,9 +496,6 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
   a.idx = g.n_r > 0 ? indices : nullptr;
   a.top_k = top_k;
   a.n_idx_groups = n_anchor_groups;
-  // d_head 128: the tcgen05 kernel gathers the borrowed rows (tile::gather4),
-  // a gathered row weighing kGatherWeight contiguous rows in the CTA split
-  const bool tc = decode_uses_tc(g.D, g.G) && (g.n_r == 0 || cache->has_tcg);
   a.gather_w = tc ? kGatherWeight : 1;
   // every retrieval item now holds min(top_k, t + 1) rows
   total = 0;

@@ -56,6 +56,9 @@ def _check_selection(sel, imp, k):
     (1, 14, 2, 1500, [0, 0], 300),
     (2, 16, 4, 257, [0, 1, 0, 1], 1000),      # top_k beyond the rows held
     (1, 8, 2, 4000, [0, 0], 1),
+    (1, 2, 2, 900, [0, 1], 100),       # one query head per group
+    (1, 8, 4, 700, [0, 0, 1, 0], 50),  # groups of 2
+    (1, 32, 2, 600, [0, 1], 128),      # groups of 16
 ])
 def test_anchor_step_selects_top_k(B, Hq, Hkv, T, labels, top_k):
     ensure_lib()
@@ -198,6 +201,8 @@ def _reuse_case(B, Hq, Hkv, D, T, S, W, labels, top_k, n_anchor, group_map, step
     (128, 14, 2, [0, 0], 97, 2, [1, 0]),
     (128, 16, 4, [0, 1, 0, 0], 5000, 1, [0, 0, 0]),   # every row borrowed: a full decode
     (64, 16, 2, [1, 0], 33, 4, [3]),
+    (128, 2, 2, [0, 1], 120, 2, [1]),            # groups of 1, gathered on the tensor cores
+    (128, 32, 2, [0, 0], 300, 2, [1, 1]),        # groups of 16
 ])
 def test_reuse_step_attends_to_borrowed_rows(D, Hq, Hkv, labels, top_k, n_anchor, gmap):
     _reuse_case(2, Hq, Hkv, D, 900, 4, 50, labels, top_k, n_anchor, gmap)
