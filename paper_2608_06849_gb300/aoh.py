@@ -169,12 +169,14 @@ def aoh_decode_step_anchor(q, k_new, v_new, cache, out, top_k, indices, stream=N
 
 def aoh_decode_step_reuse(q, k_new, v_new, cache, out, indices, top_k, group_map, stream=None):
     """H2Share reuse step; indices [B, n_anchor_groups, top_k] int32 CUDA tensor
-    from the anchor step; group_map: host list, one anchor group per
-    retrieval KV head of this layer."""
+    from the anchor step (None when the layer has no retrieval head);
+    group_map: host list, one anchor group per retrieval KV head of this
+    layer."""
     gm = (ctypes.c_int32 * max(1, len(group_map)))(*[int(x) for x in group_map])
+    n_anchor = int(indices.shape[1]) if indices is not None else 1
     _check(load().aoh_decode_step_reuse(_ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), cache,
                                         _ptr(out, "out"), _ptr(indices, "indices", torch.int32),
-                                        int(indices.shape[1]), int(top_k), gm, _stream_ptr(stream)))
+                                        n_anchor, int(top_k), gm, _stream_ptr(stream)))
 
 
 def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream=None):

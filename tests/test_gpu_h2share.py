@@ -300,6 +300,34 @@ def test_anchor_then_reuse():
     reuse.close()
 
 
+@pytest.mark.parametrize("D", [128, 64])
+def test_reuse_step_without_retrieval_heads_is_a_decode_step(D):
+    """All KV heads streaming: no list is borrowed, and the reuse step
+    equals a plain decode step on an identical cache (bit for bit: the same
+    kernel and split)."""
+    ensure_lib()
+    B, Hq, Hkv, T, S, W = 2, 8, 2, 300, 4, 50
+    labels = [1, 1]
+    c1, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, 1, 91)
+    c2 = aoh.Cache(B, Hq, Hkv, D, T + 1, S, W, labels)
+    c2.prefill(None, k, v, None)
+    wl = Workload("no-retrieval", B, Hq, Hkv, D, T, 1, S, W, 2, seed=13)
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    o1, o2 = torch.empty_like(dq), torch.empty_like(dq)
+    c1.decode_step_reuse(dq, dk, dv, o1, None, 16, [])
+    c2.decode_step(dq, dk, dv, o2)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2)
+    for b in range(B):
+        kk = np.concatenate([f64(k[b]), f64(dk[b])[None]])
+        vv = np.concatenate([f64(v[b]), f64(dv[b])[None]])
+        want = oatt.decode_step(f64(dq[b]), kk, vv, labels, S, W)
+        mag = oatt.decode_step(f64(dq[b]), kk, np.abs(vv), labels, S, W)
+        assert_matches(f64(o1[b]), want, f"no-retrieval reuse b={b}", mag)
+    c1.close()
+    c2.close()
+
+
 def test_reuse_rejects_bad_maps():
     ensure_lib()
     cache, _, _ = _filled_cache(1, 8, 2, 128, 64, 4, 16, [0, 1], 1, 71)

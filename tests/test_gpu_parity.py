@@ -31,6 +31,7 @@ CASES = {
     "group2_d128": (1, 4, 2, 128, 150, 3, 20, [1, 0], None, 3),
     "group8_d64": (1, 16, 2, 64, 200, 5, 33, [0, 1], None, 3),
     "group7_d64": (1, 7, 1, 64, 129, 2, 50, [1], None, 3),
+    "group2_d64": (1, 4, 2, 64, 150, 3, 20, [0, 1], None, 3),
     "ring_wraps_many_times": (1, 8, 2, 128, 40, 3, 5, [1, 0], None, 30),
     "single_token_prefill": (3, 8, 2, 128, 1, 4, 4, [0, 1], None, 6),
     "tile_edges": (1, 8, 2, 128, 65, 1, 63, [1, 0], None, 70),
