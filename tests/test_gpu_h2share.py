@@ -328,6 +328,73 @@ def test_reuse_step_without_retrieval_heads_is_a_decode_step(D):
     c2.close()
 
 
+def test_anchor_step_without_retrieval_heads_is_a_decode_step():
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W = 2, 8, 2, 128, 300, 4, 50
+    labels = [1, 1]
+    c1, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, 1, 93)
+    c2 = aoh.Cache(B, Hq, Hkv, D, T + 1, S, W, labels)
+    c2.prefill(None, k, v, None)
+    wl = Workload("no-retrieval-anchor", B, Hq, Hkv, D, T, 1, S, W, 2, seed=14)
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    o1, o2 = torch.empty_like(dq), torch.empty_like(dq)
+    c1.decode_step_anchor(dq, dk, dv, o1, 8, None)
+    c2.decode_step(dq, dk, dv, o2)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2)
+    assert c1.lens() == c2.lens() == [T + 1] * B
+    c1.close()
+    c2.close()
+
+
+def test_chunked_prefill_then_anchor_and_reuse():
+    """A cache filled by two prefill chunks, then an anchor step and a reuse
+    step (on a second layer's cache filled the same way) at the same
+    position: the reuse output follows the anchor's selection."""
+    ensure_lib()
+    B, Hq, Hkv, D, S, W, top_k = 1, 8, 2, 128, 4, 64, 96
+    labels = [0, 1]
+    g = Hq // Hkv
+    chunks = [700, 333]
+    T = sum(chunks)
+    caches, ks, vs = [], [], []
+    for layer in range(2):
+        cache = aoh.Cache(B, Hq, Hkv, D, T + 1, S, W, labels)
+        k = randn_bf16((B, T, Hkv, D), 300 + 2 * layer, "cuda")
+        v = randn_bf16((B, T, Hkv, D), 301 + 2 * layer, "cuda")
+        q = randn_bf16((B, T, Hq, D), 350 + layer, "cuda")
+        off = 0
+        for c in chunks:
+            out = torch.empty(B, c, Hq, D, dtype=torch.bfloat16, device="cuda")
+            cache.prefill(q[:, off:off + c].contiguous(), k[:, off:off + c].contiguous(),
+                          v[:, off:off + c].contiguous(), out)
+            off += c
+        caches.append(cache)
+        ks.append(k)
+        vs.append(v)
+    wa = Workload("chunk-anchor", B, Hq, Hkv, D, T, 1, S, W, 1, seed=15)
+    wr = Workload("chunk-reuse", B, Hq, Hkv, D, T, 1, S, W, 1, seed=16)
+    qa, ka, va = decode_inputs(wa, 0, device="cuda")
+    qr, kr, vr = decode_inputs(wr, 0, device="cuda")
+    idx = torch.empty((B, 1, top_k), dtype=torch.int32, device="cuda")
+    oa, orr = torch.empty_like(qa), torch.empty_like(qr)
+    caches[0].decode_step_anchor(qa, ka, va, oa, top_k, idx)
+    caches[1].decode_step_reuse(qr, kr, vr, orr, idx, top_k, [0])
+    torch.cuda.synchronize()
+    sel = idx.cpu().numpy()[0, 0]
+    kk0 = np.concatenate([f64(ks[0][0]), f64(ka[0])[None]])
+    _check_selection(sel, ohs.group_importance(f64(qa[0])[:g], kk0[:, 0]), top_k)
+    kk = np.concatenate([f64(ks[1][0]), f64(kr[0])[None]])
+    vv = np.concatenate([f64(vs[1][0]), f64(vr[0])[None]])
+    q = f64(qr[0])
+    want = ohs.sparse_attend(q[:g], kk[:, 0], vv[:, 0], sel)
+    mag = ohs.sparse_attend(q[:g], kk[:, 0], np.abs(vv[:, 0]), sel)
+    assert_matches(f64(orr[0, :g]), want, "reuse after chunked prefill", mag)
+    for c in caches:
+        c.check()
+        c.close()
+
+
 def test_reuse_rejects_bad_maps():
     ensure_lib()
     cache, _, _ = _filled_cache(1, 8, 2, 128, 64, 4, 16, [0, 1], 1, 71)
