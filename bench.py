@@ -19,6 +19,7 @@ import argparse
 import json
 import math
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -540,6 +541,22 @@ class OracleDecodeSample:
                 f"scaled x{self.scale}; numpy default BLAS threading")
 
 
+def host_cpu():
+    """The host CPU as the kernel reports it, and the BLAS threads numpy may use."""
+    model = platform.machine()
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                key = line.split(":")[0].strip().lower()
+                if key in ("model name", "cpu part"):
+                    model += " " + line.split(":", 1)[1].strip()
+                    break
+    except OSError:
+        pass
+    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS") or "default (one per core)"
+    return {"cpu": model, "blas_threads": threads}
+
+
 def oracle_decode_sample(budget_s=15.0):
     s = OracleDecodeSample()
     s.step_us()
@@ -548,7 +565,7 @@ def oracle_decode_sample(budget_s=15.0):
     while not vals or time.perf_counter() - t0 < budget_s:
         vals.append(s.step_us())
     return {"value": round(statistics.median(vals), 1), "unit": "us/step", "cores": os.cpu_count(),
-            "kind": "oracle", "sample": s.describe(len(vals))}
+            "kind": "oracle", "sample": s.describe(len(vals)), **host_cpu()}
 
 
 def run_reference(args):
@@ -578,7 +595,7 @@ def run_reference(args):
         "config": {"workload": f"{wl.name}: B={wl.batch} Hq={wl.n_q_heads} Hkv={wl.n_kv_heads} d={wl.d_head} "
                                f"ctx={wl.prefill_len} streaming={sum(labels)}/{len(labels)} S={wl.sink} W={wl.window}"},
         "cpu_baseline": {"value": round(value, 1), "unit": "us/step", "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": s.describe(len(vals))},
+                         "sample": s.describe(len(vals)), **host_cpu()},
         "e2e": {"value": round(value, 1), "unit": "us/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -756,7 +773,7 @@ def run_classify(args):
                      "note": "Gram flops (2 d_head^2 d_model per projection) over the whole model call; "
                              "FP64 nominal"},
         "cpu_baseline": {"value": round(cpu_s * 1e3, 1), "unit": "ms/layer", "cores": os.cpu_count(),
-                         "kind": "oracle", "sample": "layer 0, float64 oracle head_scores"}}))
+                         "kind": "oracle", "sample": "layer 0, float64 oracle head_scores", **host_cpu()}}))
 
 
 def run_h2map(args):
@@ -815,7 +832,8 @@ def run_h2map(args):
                              "Grams) over the whole call's time, including workspace allocation, the fp64 trace "
                              "kernel and the host copies; " + note + " burst peak"},
         "cpu_baseline": {"value": round(cpu_s * 1e3, 1), "unit": "ms/layer pair", "cores": os.cpu_count(),
-                         "kind": "oracle", "sample": "the same layer pair, float64 oracle group_similarity"}}))
+                         "kind": "oracle", "sample": "the same layer pair, float64 oracle group_similarity",
+                         **host_cpu()}}))
 
 
 def main():
