@@ -49,3 +49,48 @@ def test_noalloc_decode_matches_handle_decode(B, Hq, Hkv, D, T, S, W, labels):
     cache.check()
     assert torch.equal(kv_copy, cache.buffer)            # the same rows were appended
     cache.close()
+
+
+def test_noalloc_decode_replays_from_a_cuda_graph():
+    """Decode steps captured once in a CUDA graph (the launch-bound inner loop
+    of a server) and replayed give the same outputs as the handle API step by
+    step; the device lengths advance on replay."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, labels = 2, 32, 8, 128, 5000, 64, 700, [1, 0, 0, 1, 1, 0, 0, 1]
+    steps = 3
+    wl = Workload("graph", B, Hq, Hkv, D, T, steps + 1, S, W, sum(labels), seed=4)
+    cache = aoh.Cache(B, Hq, Hkv, D, T + steps + 2, S, W, labels)
+    k = randn_bf16((B, T, Hkv, D), 21, "cuda")
+    v = randn_bf16((B, T, Hkv, D), 22, "cuda")
+    cache.prefill(None, k, v, None)
+    torch.cuda.synchronize()
+    kv_copy = cache.buffer.clone()
+    lens = torch.full((B,), T, dtype=torch.int32, device="cuda")
+    inputs = [decode_inputs(wl, s, device="cuda") for s in range(steps + 1)]
+    # step 0 outside the graph: the first call sets the library up (symbol
+    # address, kernel attributes)
+    ref0 = torch.empty_like(inputs[0][0])
+    na0 = torch.empty_like(inputs[0][0])
+    cache.decode_step(*inputs[0], ref0)
+    aoh.aoh_decode_step_noalloc(cache.cfg, labels, kv_copy, lens, T, *inputs[0], na0)
+    torch.cuda.synchronize()
+    outs = [torch.full_like(inputs[0][0], float("nan")) for _ in range(steps)]
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for s in range(steps):
+            aoh.aoh_decode_step_noalloc(cache.cfg, labels, kv_copy, lens, T + 1 + s, *inputs[s + 1], outs[s])
+    torch.cuda.synchronize()
+    assert lens.tolist() == [T + 1] * B            # capture ran nothing
+    graph.replay()
+    torch.cuda.synchronize()
+    assert lens.tolist() == [T + 1 + steps] * B
+    for s in range(steps):
+        ref = torch.empty_like(outs[s])
+        cache.decode_step(*inputs[s + 1], ref)
+        torch.cuda.synchronize()
+        assert torch.isfinite(outs[s].float()).all()
+        err = (outs[s].float() - ref.float()).abs()
+        assert err.max().item() <= MAX_ABS, (s, err.max().item())
+        assert err.mean().item() <= MEAN_ABS, (s, err.mean().item())
+    assert torch.equal(kv_copy, cache.buffer)
+    cache.close()
