@@ -716,6 +716,86 @@ def run_stack(args):
         "peak_note": note}))
 
 
+def run_graph(args):
+    """Batch-1 decode latency per token through a whole Qwen2.5-7B-shaped
+    model (28 layers of 28 query / 4 KV heads, d_head 128, 2 of 4 KV heads
+    streaming, S=128, W=4096; one cache per layer, seeded N(0,1) bf16 K/V)
+    at several context lengths, as the paper reports it. Each token runs the
+    28 layers' decode steps through the allocation-free entry point, once
+    launched eagerly from the host and once replayed as one CUDA graph
+    captured for all 28 layers."""
+    import torch
+
+    from paper_2608_06849_gb300 import aoh
+    from paper_2608_06849_gb300 import build as aoh_build
+    from paper_2608_06849_gb300.workloads import STACK_256K, decode_inputs, labels_for, randn_bf16
+    aoh_build.build()
+    aoh.load()
+    peaks, note = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    wl = STACK_256K
+    L, B, Hq, Hkv, D = wl.layers, 1, wl.n_q_heads, wl.n_kv_heads, wl.d_head
+    tokens = max(args.steps, 8)
+    points = []
+    for T in (4096, 32768, 131072):
+        cap = T + 2 * tokens + args.warmup + 8
+        caches, lens, ins, outs, labels = [], [], [], [], []
+        for layer in range(L):
+            lab = labels_for(wl, layer=layer)
+            c = aoh.Cache(B, Hq, Hkv, D, cap, wl.sink, wl.window, lab)
+            k = randn_bf16((B, T, Hkv, D), 5000 + 2 * layer, "cuda")
+            v = randn_bf16((B, T, Hkv, D), 5001 + 2 * layer, "cuda")
+            c.prefill(None, k, v, None)
+            del k, v
+            caches.append(c)
+            labels.append(lab)
+            lens.append(torch.full((B,), T, dtype=torch.int32, device="cuda"))
+            ins.append(decode_inputs(wl, layer, device="cuda"))
+            outs.append(torch.empty(B, Hq, D, dtype=torch.bfloat16, device="cuda"))
+        torch.cuda.synchronize()
+        bound = cap - 1  # host upper bound of every length during this run
+
+        def token():
+            for layer in range(L):
+                aoh.aoh_decode_step_noalloc(caches[layer].cfg, labels[layer], caches[layer].buffer, lens[layer], bound,
+                                            *ins[layer], outs[layer])
+
+        for _ in range(max(args.warmup, 3)):
+            token()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(tokens):
+            token()
+        e1.record()
+        torch.cuda.synchronize()
+        eager_us = e0.elapsed_time(e1) * 1000 / tokens
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            token()
+        graph.replay()
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(tokens):
+            graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        graph_us = e0.elapsed_time(e1) * 1000 / tokens
+        t_mid = T + max(args.warmup, 3) + tokens
+        nbytes = sum(decode_bytes([t_mid], labels[layer], wl) for layer in range(L))
+        points.append({"context": T, "eager_us_per_token": round(eager_us, 1), "graph_us_per_token": round(graph_us, 1),
+                       "bytes_per_token": nbytes, "graph_hbm_gbs": round(nbytes / (graph_us * 1e-6) / 1e9, 1),
+                       "graph_frac_of_peak": round(nbytes / (graph_us * 1e-6) / 1e9 / hbm, 4)})
+        for c in caches:
+            c.close()
+        del caches, lens, ins, outs, graph
+        torch.cuda.empty_cache()
+    print(json.dumps({
+        "workload": f"{wl.name}-decode-per-token: {L} layers x (Hq={Hq} Hkv={Hkv} d={D}), B=1, 2 of 4 KV heads "
+                    f"streaming per layer, S={wl.sink} W={wl.window}; {tokens} tokens per point",
+        "points": points, "peak_hbm_gbs": hbm, "peak_note": note}))
+
+
 def run_classify(args):
     """Effective-rank classification of a Qwen2.5-7B-shaped model (28 layers
     of 28 query / 4 KV heads, d_head 128, d_model 3584; seeded N(0,1) bf16
@@ -844,9 +924,11 @@ def main():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--prefill-steps", type=int, default=10)
     ap.add_argument("--prefill-chunks", type=int, default=8)
-    ap.add_argument("--workload", choices=["default", "ragged", "stack", "classify", "h2map"], default="default",
+    ap.add_argument("--workload", choices=["default", "ragged", "stack", "classify", "h2map", "graph"],
+                    default="default",
                     help="default: the headline decode + prefill run; ragged / stack: the other two workloads; "
-                         "classify: the effective-rank head classifier; h2map: the H2Share head mapping")
+                         "classify: the effective-rank head classifier; h2map: the H2Share head mapping; "
+                         "graph: batch-1 per-token decode through 28 layers, eager and as one CUDA graph")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--h2-top-k", type=int, default=2048, help="positions an H2Share anchor step selects")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -866,6 +948,8 @@ def main():
         run_classify(args)
     elif args.workload == "h2map":
         run_h2map(args)
+    elif args.workload == "graph":
+        run_graph(args)
     else:
         run_native(args)
 
