@@ -418,9 +418,10 @@ def run_native(args):
     del chunks, couts
 
     # ---------------- cpu baseline (oracle on a bounded sample), rank 0 only
-    cpu = None
+    cpu = pcpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = oracle_decode_sample(args.cpu_seconds)
+        pcpu = oracle_prefill_sample(min(10.0, args.cpu_seconds))
 
     if rank != 0:
         return
@@ -458,7 +459,8 @@ def run_native(args):
                     "roofline": {"bound": "tensor", "achieved": round(pre_tflops, 2), "peak": tf_peak,
                                  "unit": "TFLOP/s", "frac": round(pre_tflops / tf_peak, 4),
                                  "traffic": traffic_for("prefill"),
-                                 "peak_note": f"{peak_note} dense bf16 (burst); time includes the cache append"}},
+                                 "peak_note": f"{peak_note} dense bf16 (burst); time includes the cache append"},
+                    "cpu_baseline": pcpu},
         "chunked_prefill": {"chunks": n_chunks, "chunk_tokens": C, "ms": round(chunk_ms, 3),
                             "tflops": round(flops / (chunk_ms * 1e-3) / 1e12, 2),
                             "note": "same 32K prefill as consecutive chunks; each chunk reads the cached prefix"},
@@ -539,6 +541,46 @@ class OracleDecodeSample:
         return (f"float64 oracle, 1 of {self.wl.batch} sequences x (1 retrieval + 1 streaming) of "
                 f"{len(self.labels)} KV head groups at ctx {self.wl.prefill_len}, median of {reps} reps, "
                 f"scaled x{self.scale}; numpy default BLAS threading")
+
+
+def oracle_prefill_sample(budget_s=10.0):
+    """The float64 oracle on seeded random query rows of the 32K prefill (all
+    28 query heads, the prefill's labels), until about budget_s has passed,
+    extrapolated to the whole prefill by attended (query, key) pairs."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from paper_2608_06849_gb300.workloads import randn_bf16
+    wl, labels = prefill_workload()
+    T, D, S, W, g = wl.prefill_len, wl.d_head, wl.sink, wl.window, wl.g
+    k = randn_bf16((T, wl.n_kv_heads, D), 9101).float().numpy().astype(np.float64)
+    v = randn_bf16((T, wl.n_kv_heads, D), 9102).float().numpy().astype(np.float64)
+    rng = np.random.default_rng(9103)
+
+    def pairs(i):
+        tot = 0
+        for lab in labels:
+            if lab == 0:
+                tot += i + 1
+            else:
+                tot += min(i + 1, S) + max(0, i - max(S, i - W + 1) + 1)
+        return tot * g
+
+    spent, done_pairs, n_rows = 0.0, 0, 0
+    while spent < budget_s:
+        rows = np.sort(rng.choice(T, size=8, replace=False))
+        q = randn_bf16((8, wl.n_q_heads, D), 9104 + n_rows).float().numpy().astype(np.float64)
+        t0 = time.perf_counter()
+        oatt.attend(q, rows, k, v, labels, S, W)
+        spent += time.perf_counter() - t0
+        done_pairs += sum(pairs(int(i)) for i in rows)
+        n_rows += 8
+    total_pairs = prefill_flops(wl, labels, T) / (4.0 * D)
+    ms = spent / done_pairs * total_pairs * 1e3
+    return {"value": round(ms, 1), "unit": "ms/prefill", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"float64 oracle on {n_rows} random query rows (all {wl.n_q_heads} heads) of the {T}-token "
+                      f"prefill, {spent:.1f} s, extrapolated by attended (query, key) pairs "
+                      f"({done_pairs} of {int(total_pairs)})", **host_cpu()}
 
 
 def host_cpu():
