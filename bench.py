@@ -543,15 +543,17 @@ class OracleDecodeSample:
                 f"scaled x{self.scale}; numpy default BLAS threading")
 
 
-def oracle_prefill_sample(budget_s=10.0):
-    """The float64 oracle on seeded random query rows of the 32K prefill (all
-    28 query heads, the prefill's labels), until about budget_s has passed,
-    extrapolated to the whole prefill by attended (query, key) pairs."""
+def oracle_prefill_sample(budget_s=10.0, wl=None, labels=None):
+    """The float64 oracle on seeded random query rows of a prefill (all query
+    heads, the workload's labels; the 32K prefill by default), until about
+    budget_s has passed, extrapolated to the whole prefill by attended
+    (query, key) pairs."""
     import numpy as np
 
     from oracle import attention as oatt
     from paper_2608_06849_gb300.workloads import randn_bf16
-    wl, labels = prefill_workload()
+    if wl is None:
+        wl, labels = prefill_workload()
     T, D, S, W, g = wl.prefill_len, wl.d_head, wl.sink, wl.window, wl.g
     k = randn_bf16((T, wl.n_kv_heads, D), 9101).float().numpy().astype(np.float64)
     v = randn_bf16((T, wl.n_kv_heads, D), 9102).float().numpy().astype(np.float64)
@@ -583,6 +585,40 @@ def oracle_prefill_sample(budget_s=10.0):
                       f"({done_pairs} of {int(total_pairs)})", **host_cpu()}
 
 
+def oracle_decode_layer(wl, labels, lens, budget_s=5.0, max_seqs=4):
+    """The float64 oracle on one layer's decode step (all heads) for up to
+    max_seqs of the batch's sequences at their lengths, repeated for about
+    budget_s; the median scaled to the whole batch by rows attended."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from paper_2608_06849_gb300.workloads import randn_bf16
+    D, S, W = wl.d_head, wl.sink, wl.window
+
+    def rows(t):
+        return sum((t + 1) if lab == 0 else min(t + 1, S + W) for lab in labels)
+
+    sample = list(lens[:max_seqs])
+    data = []
+    for i, t in enumerate(sample):
+        k = randn_bf16((t + 1, wl.n_kv_heads, D), 9201 + 3 * i).float().numpy().astype(np.float64)
+        v = randn_bf16((t + 1, wl.n_kv_heads, D), 9202 + 3 * i).float().numpy().astype(np.float64)
+        q = randn_bf16((wl.n_q_heads, D), 9203 + 3 * i).float().numpy().astype(np.float64)
+        data.append((q, k, v))
+    vals = []
+    t0 = time.perf_counter()
+    while not vals or time.perf_counter() - t0 < budget_s:
+        a = time.perf_counter()
+        for q, k, v in data:
+            oatt.decode_step(q, k, v, labels, S, W)
+        vals.append(time.perf_counter() - a)
+    scale = sum(rows(t) for t in lens) / sum(rows(t) for t in sample)
+    return {"value": round(statistics.median(vals) * scale * 1e6, 1), "unit": "us/step", "cores": os.cpu_count(),
+            "kind": "oracle", "sample": f"float64 oracle decode step on {len(sample)} of {len(lens)} sequences "
+                                        f"(all heads), median of {len(vals)} reps, scaled x{scale:.2f} by rows "
+                                        f"attended", **host_cpu()}
+
+
 def host_cpu():
     """The host CPU as the kernel reports it, and the BLAS threads numpy may use."""
     model = platform.machine()
@@ -591,7 +627,9 @@ def host_cpu():
             for line in f:
                 key = line.split(":")[0].strip().lower()
                 if key in ("model name", "cpu part"):
-                    model += " " + line.split(":", 1)[1].strip()
+                    val = line.split(":", 1)[1].strip()
+                    # Arm reports a part number; 0xd4f is the Neoverse V2 (Grace)
+                    model += " " + {"0xd4f": "Neoverse-V2 (0xd4f)"}.get(val, val)
                     break
     except OSError:
         pass
@@ -699,7 +737,12 @@ def run_ragged(args):
     print(json.dumps({"workload": f"{RAGGED.name}: B={B} Hq={RAGGED.n_q_heads} Hkv={Hkv} d={D} "
                                   f"lens uniform [4096, 32768] seed {RAGGED.seed} S={RAGGED.sink}",
                       "metric": "decode attn us/step and HBM GB/s", "steps": args.steps, "warmup": args.warmup,
-                      "peak_hbm_gbs": hbm, "peak_note": note, "sweep": points}))
+                      "peak_hbm_gbs": hbm, "peak_note": note, "sweep": points,
+                      "cpu_baseline": None if args.no_cpu_baseline else dict(
+                          oracle_decode_layer(dataclasses.replace(RAGGED, n_streaming=Hkv // 2, window=2048),
+                                              labels_for(dataclasses.replace(RAGGED, n_streaming=Hkv // 2)),
+                                              list(lens), budget_s=5.0),
+                          point="streaming_frac 0.5, window 2048")}))
 
 
 def run_stack(args):
@@ -755,7 +798,10 @@ def run_stack(args):
         "stack_estimate": {"prefill_s": round(wl.layers * pre_ms / 1000, 3),
                            "decode_ms_per_token": round(wl.layers * us / 1000, 3)},
         "kv_bytes_stack": kv_aoh, "kv_bytes_all_retrieval": kv_full, "kv_ratio": round(kv_full / kv_aoh, 4),
-        "peak_note": note}))
+        "peak_note": note,
+        "cpu_baseline": None if args.no_cpu_baseline else {
+            "decode": oracle_decode_layer(wl, labels, before, budget_s=5.0),
+            "prefill": oracle_prefill_sample(8.0, wl, labels)}}))
 
 
 def run_graph(args):
