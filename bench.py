@@ -997,8 +997,8 @@ def run_h2map(args):
         "roofline": {"bound": "tensor", "achieved": round(ach, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(ach / peak, 4),
                      "note": "bf16 contraction flops of the whole call (Q_a Q_r^T, K_r K_a^T, four diagonal-block "
-                             "Grams) over the whole call's time, including workspace allocation, the fp64 trace "
-                             "kernel and the host copies; " + note + " burst peak"},
+                             "Grams) over the whole call's time, including the fp64 trace kernel, the map kernel "
+                             "and the host copy; " + note + " burst peak"},
         "cpu_baseline": {"value": round(cpu_s * 1e3, 1), "unit": "ms/layer pair", "cores": os.cpu_count(),
                          "kind": "oracle", "sample": "the same layer pair, float64 oracle group_similarity",
                          **host_cpu()}}))

@@ -218,9 +218,10 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
  *                  group_map of aoh_decode_step_reuse.
  *   group_sim_out  host double [n_kv_heads][n_kv_heads] (anchor-major), or NULL.
  * The d_model contractions run on the tensor cores (bf16 in, fp32
- * accumulate); traces and norms in fp64. Allocates temporary device memory
- * stream-ordered and synchronises `stream`. Errors: INVALID, UNSUPPORTED,
- * TIMEOUT, CUDA.
+ * accumulate); traces and norms in fp64. Keeps one device workspace per
+ * device for the process (allocated with cudaMalloc on the first call that
+ * needs more; calls on a device are serialised) and synchronises `stream`.
+ * Errors: INVALID, UNSUPPORTED, TIMEOUT, CUDA.
  */
 aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_anchor, const void* w_q_reuse,
                            const void* w_k_reuse, int32_t n_q_heads, int32_t n_kv_heads, int32_t d_head,

@@ -33,6 +33,9 @@
 #include <math.h>
 
 #include <algorithm>
+#include <cstring>
+#include <mutex>
+#include <vector>
 
 #include "../../include/aoh.h"
 #include "common.cuh"
@@ -302,6 +305,15 @@ __global__ void map_kernel(const double* num, const double* na, const double* nr
   }
 }
 
+// One workspace per device, grown on demand and kept for the process (a
+// stream-ordered allocation per call would be mapped and released at every
+// synchronise); calls on one device are serialised by the mutex, and each
+// synchronises its stream before returning, so the next may reuse it.
+constexpr int kWsDevices = 64;
+std::mutex g_ws_mutex;
+void* g_ws[kWsDevices] = {};
+size_t g_ws_cap[kWsDevices] = {};
+
 }  // namespace
 }  // namespace aoh
 
@@ -338,9 +350,19 @@ extern "C" aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_an
   // head and group similarities; map; error word
   const size_t bytes = 3 * (size_t)nk * nk * 4 + ((size_t)Hq * Hq + 2 * Hq) * 8 + 2 * (size_t)Hq * 8 +
                        (size_t)Hq * Hq * 8 + (size_t)Hkv * Hkv * 8 + Hkv * 4 + 256;
-  void* ws = nullptr;
-  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
-  if (e != cudaSuccess) return fail(AOH_ERR_CUDA, "aoh_h2share_map: cudaMallocAsync failed");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kWsDevices) return fail(AOH_ERR_CUDA, "aoh_h2share_map: no usable device");
+  std::lock_guard<std::mutex> lock(g_ws_mutex);
+  if (g_ws_cap[dev] < bytes) {
+    if (g_ws[dev]) cudaFree(g_ws[dev]);
+    g_ws[dev] = nullptr;
+    g_ws_cap[dev] = 0;
+    e = cudaMalloc(&g_ws[dev], bytes);
+    if (e != cudaSuccess) return fail(AOH_ERR_CUDA, "aoh_h2share_map: workspace allocation failed");
+    g_ws_cap[dev] = bytes;
+  }
+  void* ws = g_ws[dev];
   float* Y = static_cast<float*>(ws);
   float* gka = Y + (size_t)nk * nk;
   float* gkr = gka + (size_t)nk * nk;
@@ -373,15 +395,16 @@ extern "C" aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_an
     map_kernel<<<1, 1024, 0, s>>>(num, na, nr, Hq, Hkv, lab, inv, sim, gsim, map);
     e = cudaGetLastError();
   }
-  uint32_t h_err = 0;
-  if (e == cudaSuccess) e = cudaMemcpyAsync(map_out, map, Hkv * 4, cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess && group_sim_out)
-    e = cudaMemcpyAsync(group_sim_out, gsim, (size_t)Hkv * Hkv * 8, cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(&h_err, err, 4, cudaMemcpyDeviceToHost, s);
-  const cudaError_t f = cudaFreeAsync(ws, s);
-  if (e == cudaSuccess) e = f;
+  // group similarities, map and error word are contiguous: one copy back
+  const size_t res_bytes = (size_t)Hkv * Hkv * 8 + (size_t)Hkv * 4 + 4;
+  std::vector<unsigned char> res(res_bytes);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(res.data(), gsim, res_bytes, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return fail(AOH_ERR_CUDA, "aoh_h2share_map: a CUDA call failed");
+  uint32_t h_err = 0;
+  memcpy(map_out, res.data() + (size_t)Hkv * Hkv * 8, (size_t)Hkv * 4);
+  if (group_sim_out) memcpy(group_sim_out, res.data(), (size_t)Hkv * Hkv * 8);
+  memcpy(&h_err, res.data() + (size_t)Hkv * Hkv * 8 + (size_t)Hkv * 4, 4);
   if (h_err) return fail(AOH_ERR_TIMEOUT, "aoh_h2share_map: a kernel's bounded wait ran out");
   return AOH_OK;
 }
