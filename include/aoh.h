@@ -165,8 +165,9 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
  *            increasing KV-head index), written on the stream; entries past
  *            min(top_k, t + 1) are -1.
  * Needs d_head 128 (the tensor-core decode). The first call allocates a
- * workspace of about B * n_r * max_seq * (group size + 1) floats in the handle
- * (a cudaMalloc, which synchronises the device); aoh_cache_destroy frees it.
+ * workspace of about B * n_r * max_seq * (group size) floats in the handle,
+ * plus B * n_r * max_seq more when max_seq exceeds 147456 (a cudaMalloc,
+ * which synchronises the device); aoh_cache_destroy frees it.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,

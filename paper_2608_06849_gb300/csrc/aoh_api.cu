@@ -127,7 +127,8 @@ struct aoh_cache {
   // prefill work list (device), grown on demand
   int4* d_work = nullptr;
   size_t work_cap = 0;
-  // H2Share anchor workspace (scores, importance), allocated on first use
+  // H2Share anchor workspace (scores, head states, importance overflow),
+  // allocated on first use
   float* d_h2 = nullptr;
 };
 
@@ -445,18 +446,16 @@ aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* 
   if (!decode_uses_tc(g.D, g.G))
     return fail(AOH_ERR_UNSUPPORTED, "the anchor step needs the d_head 128 tensor-core decode");
   if (g.n_r > 0 && !cache->d_h2) {
-    // scores [B][n_r][G][max_seq], importance, chunk states, histograms
+    // scores [B][n_r][G][max_seq padded to 4], head states, importance overflow
     const size_t n = h2_workspace_floats(g.B, g.n_r, g.G, g.max_seq);
     cudaError_t e = cudaMalloc(&cache->d_h2, n * sizeof(float));
-    if (e == cudaSuccess) e = h2_workspace_clear(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, (cudaStream_t)stream);
     if (e != cudaSuccess) {
       if (cache->d_h2) cudaFree(cache->d_h2);
       cache->d_h2 = nullptr;
       return cuda_fail(e, "anchor workspace allocation");
     }
   }
-  if (g.n_r > 0) h2_decode_outputs(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, &a.scores, &a.score_stats);
-  a.score_stride = g.max_seq;
+  if (g.n_r > 0) h2_decode_outputs(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, &a.scores, &a.score_stride, &a.score_stats);
   a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e = launch_decode(a, s);

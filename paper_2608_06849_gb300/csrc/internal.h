@@ -136,14 +136,15 @@ cudaError_t launch_decode_cc(const DecodeArgs& a, cudaStream_t s);
 int decode_cc_ctas(long long total_rows, int num_sms);
 bool decode_cc_supported(int D, int G);
 // H2Share anchor selection after a decode step that wrote its scores to
-// the start of `ws` ([B][n_r][G][max_seq] floats): per (sequence, retrieval
+// the start of `ws` ([B][n_r][G][stride] floats): per (sequence, retrieval
 // head) the top_k positions by group importance. `ws` holds
 // h2_workspace_floats() floats.
 size_t h2_workspace_floats(int B, int n_r, int G, int max_seq);
-// Where the decode kernel writes the scores and per-head states in `ws`.
-void h2_decode_outputs(float* ws, int B, int n_r, int G, int max_seq, float** scores, float2** stats);
-// Zero the histograms of a new workspace (the select kernel keeps them zero).
-cudaError_t h2_workspace_clear(float* ws, int B, int n_r, int G, int max_seq, cudaStream_t s);
+// Where the decode kernel writes the scores (row stride `stride`, max_seq
+// rounded up to a multiple of 4) and the per-head states in `ws`.
+void h2_decode_outputs(float* ws, int B, int n_r, int G, int max_seq, float** scores, int* stride, float2** stats);
+// One cluster launch computes the importances and selects; `lens` holds the
+// lengths after the anchor step's append.
 cudaError_t launch_h2_topk(float* ws, int max_seq, const int32_t* lens, int B, int n_r, int G, int top_k,
                            int32_t* idx_out, cudaStream_t s);
 // CTAs for a decode launch over `total_rows` cached rows on `num_sms` SMs

@@ -59,6 +59,7 @@ def _check_selection(sel, imp, k):
     (1, 2, 2, 900, [0, 1], 100),       # one query head per group
     (1, 8, 4, 700, [0, 0, 1, 0], 50),  # groups of 2
     (1, 32, 2, 600, [0, 1], 128),      # groups of 16
+    (1, 8, 2, 5, [0, 1], 2),           # one slice holds every row, the others none
 ])
 def test_anchor_step_selects_top_k(B, Hq, Hkv, T, labels, top_k):
     ensure_lib()
@@ -138,6 +139,54 @@ def test_anchor_selection_with_one_crowded_bucket():
     # the tied positions are taken lowest first
     tied = sel[sel < T]
     assert np.array_equal(tied[: len(tied)], np.arange(len(tied))) or imp[T] < imp[0]
+
+
+def test_anchor_selection_past_the_shared_memory_slices():
+    """200K cached rows: each of a cluster's eight slices holds more rows
+    than its CTA keeps in shared memory, so the rest of the importances go
+    through global memory."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, top_k, steps = 1, 8, 2, 128, 200000, 4, 64, 2048, 2
+    labels = [0, 1]
+    g = Hq // Hkv
+    cache, k, v = _filled_cache(B, Hq, Hkv, D, T, S, W, labels, steps, 131)
+    wl = Workload("long", B, Hq, Hkv, D, T, steps, S, W, 1, seed=13)
+    kall = f64(k[0])
+    for step in range(steps):
+        dq, dk, dv = decode_inputs(wl, step, device="cuda")
+        idx = torch.full((B, 1, top_k), -7, dtype=torch.int32, device="cuda")
+        cache.decode_step_anchor(dq, dk, dv, torch.empty_like(dq), top_k, idx)
+        torch.cuda.synchronize()
+        kall = np.concatenate([kall, f64(dk[0])[None]])
+        imp = ohs.group_importance(f64(dq[0])[:g], kall[:, 0])
+        _check_selection(idx.cpu().numpy()[0, 0], imp, top_k)
+    cache.close()
+
+
+def test_anchor_selection_ties_across_slices_and_overflow():
+    """180K identical keys: every cached row ties, and the top_k rows are
+    the lowest positions, taken across several slices and past the rows a
+    CTA keeps in shared memory."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, top_k = 1, 8, 2, 128, 180000, 4, 64, 100000
+    labels = [0, 1]
+    g = Hq // Hkv
+    cache = aoh.Cache(B, Hq, Hkv, D, T + 1, S, W, labels)
+    k = randn_bf16((B, 1, Hkv, D), 141, "cuda").expand(B, T, Hkv, D).contiguous()
+    v = randn_bf16((B, T, Hkv, D), 142, "cuda")
+    cache.prefill(None, k, v, None)
+    wl = Workload("ties", B, Hq, Hkv, D, T, 1, S, W, 1, seed=14)
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    idx = torch.full((B, 1, top_k), -7, dtype=torch.int32, device="cuda")
+    cache.decode_step_anchor(dq, dk, dv, torch.empty_like(dq), top_k, idx)
+    torch.cuda.synchronize()
+    sel = idx.cpu().numpy()[0, 0]
+    kk = np.concatenate([f64(k[0]), f64(dk[0])[None]])
+    imp = ohs.group_importance(f64(dq[0])[:g], kk[:, 0])
+    _check_selection(sel, imp, top_k)
+    tied = sel[sel < T]
+    want = top_k if imp[T] < imp[0] else top_k - 1
+    assert len(tied) == want and np.array_equal(tied, np.arange(want))
     cache.close()
 
 
