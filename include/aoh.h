@@ -299,14 +299,14 @@ const char* aoh_last_error(void);
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress, with that device current) and caches it; make
  *     that first call before any stream capture.
- *   - Every call shares the one array and leaves its contents behind; the
- *     counters that must start at zero are cleared on the stream at the start
- *     of each call. Calls whose kernels overlap on the GPU (on different
- *     streams, or from different threads without ordering) race on the
- *     scratch and produce wrong results: order them on one stream.
- *   - A bounded-wait timeout inside the kernel is recorded only in the
- *     scratch error word, which this call does not report; the outputs of
- *     such a call are unspecified.
+ *   - Every call shares the one array. Each call is a single kernel launch,
+ *     which leaves the counters that must start at zero at zero when it
+ *     ends. Calls whose kernels overlap on the GPU (on different streams, or
+ *     from different threads without ordering) race on the scratch and
+ *     produce wrong results: order them on one stream.
+ *   - A bounded-wait timeout inside the kernel is not reported by this call
+ *     and leaves the outputs of that call unspecified; the launch still
+ *     leaves the scratch clean for the next call.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,

@@ -328,12 +328,20 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
 }
 
 // The launch's last CTA advances every sequence length by one. Called by
-// thread 0 after a __syncthreads that follows all of the CTA's work.
+// thread 0 after a __syncthreads that follows all of the CTA's work. A
+// completed merge leaves its counters at zero; after a timeout some may be
+// left behind, and a self-cleaning launch zeroes them and the error word.
 __device__ __forceinline__ void finish_launch(const DecodeArgs& a) {
   __threadfence();
   const uint32_t prev = atomicAdd(a.done, 1u);
   if (prev == gridDim.x - 1) {
     for (int i = 0; i < a.geom.B; ++i) a.lens[i] += 1;
+    if (a.self_clean && *reinterpret_cast<volatile uint32_t*>(a.err) != 0u) {
+      const int items = a.geom.B * (a.geom.n_r + a.geom.n_s);
+      for (int i = 0; i < items; ++i) a.counters[i] = 0u;
+      for (int i = 0; i < 2 * (int)gridDim.x; ++i) a.gcounters[i] = 0u;
+      *a.err = 0u;
+    }
     __threadfence();
     *a.done = 0u;
   }

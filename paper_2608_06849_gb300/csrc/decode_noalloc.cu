@@ -134,10 +134,11 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   const int cap_ctas = (int)(kNoAllocPartialBytes / (decode_partial_floats(1, G, c.d_head) * 4));
   if (n_ctas > cap_ctas) n_ctas = cap_ctas;
   if (n_ctas > kNoAllocMaxCtas) n_ctas = kNoAllocMaxCtas;
-  // err, done and the arrival counters must start at zero; clear them every call.
-  e = cudaMemsetAsync(header, 0, (size_t)(64 + items + 2 * n_ctas) * 4, s);
-  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cudaMemsetAsync failed");
-
+  // err, done and the arrival counters start at zero: the array is
+  // zero-initialised, and every launch leaves them at zero (self-cleaning,
+  // timeouts included), so consecutive calls need no clearing launch and
+  // each decode launch overlaps the previous one's tail (programmatic
+  // dependent launch).
   DecodeArgs a;
   if (!make_cache_region_maps(&a.tcr, &a.tcs, g, kv_buffer))
     return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: cuTensorMapEncodeTiled failed");
@@ -154,6 +155,7 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   a.gcounters = header + 64 + items;
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
   a.n_ctas = n_ctas;
+  a.self_clean = 1;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));
   e = launch_decode(a, s);
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: kernel launch failed");

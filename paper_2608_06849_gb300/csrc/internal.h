@@ -61,6 +61,10 @@ struct DecodeArgs {
   uint32_t* done;     // CTAs finished in this launch
   uint32_t* err;      // error word
   int n_ctas;         // CTAs sharing the rows of all items equally
+  // nonzero: the launch's last CTA also leaves the error word and every
+  // counter at zero after a timed-out launch, so the next launch needs no
+  // clearing (the allocation-free entry point, which reports no timeouts)
+  int self_clean = 0;
   float scale_log2;   // log2(e) / sqrt(D)
   // H2Share anchor step (tcgen05 kernel): when non-null, every retrieval row's
   // scores (log2 units) go to scores[((b * n_r + i) * G + h) * score_stride + row],
