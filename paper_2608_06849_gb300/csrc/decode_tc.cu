@@ -169,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
     // Retrieval items of the H2Share reuse step (a.idx): every lane gathers
     // four of a tile's 128 borrowed rows (tile::gather4 over the gather map,
     // one instruction per row quad, 64-column half and K or V), with the
-    // tile's indices loaded one tile ahead. Slots past the item's rows read
+    // tile's indices loaded two tiles ahead. Slots past the item's rows read
     // row 0 (the softmax gives them zero weight); slots holding the new
     // token (position t, not in the cache yet) read row 0 too and are
     // listed in the stage's patch mask for the MMA warp to overwrite.
@@ -192,9 +192,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
         const int32_t* rowlist = a.idx + ((size_t)b * a.n_idx_groups + a.idx_map[k]) * a.top_k;
         const int t = dec::seq_len(a, b, ls);
         const int kbase = region * 2 * g.max_seq, vbase = kbase + g.max_seq;
-        int nxt[4];
+        // indices of this tile (nxt) and the next (nx2): each tile's loads
+        // are issued two tiles before its gathers
+        int nxt[4], nx2[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) nxt[j] = lo + 4 * lane + j < hi ? __ldg(rowlist + lo + 4 * lane + j) : 0;
+        for (int j = 0; j < 4; ++j) {
+          const int j0 = lo + 4 * lane + j;
+          nxt[j] = j0 < hi ? __ldg(rowlist + j0) : 0;
+          nx2[j] = j0 + kBN < hi ? __ldg(rowlist + j0 + kBN) : 0;
+        }
         for (int row0 = lo; row0 < hi; row0 += kBN) {
           int cr[4];
           uint32_t newrow[4];
@@ -204,8 +210,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
             const int c = min(max(nxt[j], 0), t);
             newrow[j] = __ballot_sync(0xffffffffu, valid && c == t);
             cr[j] = valid && c != t ? c : 0;
-            const int jn = row0 + kBN + 4 * lane + j;
-            if (jn < hi) nxt[j] = __ldg(rowlist + jn);
+            nxt[j] = nx2[j];
+            const int jn = row0 + 2 * kBN + 4 * lane + j;
+            if (jn < hi) nx2[j] = __ldg(rowlist + jn);
           }
           const int st = it % kNS;
           int go = 1;
