@@ -20,17 +20,20 @@
 //      every CTA adds its nonzero bins into CTA 0's histogram with remote
 //      shared-memory atomics; one warp of CTA 0 picks the bucket and sends
 //      (digit, rank) back.
-//   3. Each warp counts its rows above that bucket and sends the bucket's
-//      members (few, as a rule) to CTA 0, which finds the exact threshold
-//      among them (two more radix levels, 11 and 10 bits), the number of
-//      rows equal to it still needed, and from these every warp's output
-//      offset and share of the equal rows, and sends each warp its share.
-//      If some CTA has more members than CTA 0 has room for, every level is
-//      instead a full pass over the slices, as in step 2, followed by an
-//      exchange of per-CTA counts.
-//   4. An ordered compaction: each warp walks its run 128 rows at a time
-//      (four per lane); ballots place the rows above the threshold and, in
-//      position order, as many rows equal to it as its share.
+//   3. Each warp lists the rows of its run at or above that bucket,
+//      (position, bits) in position order, and counts those above it; the
+//      listed rows not above it are the bucket's members (few, as a rule),
+//      which go to CTA 0. CTA 0 finds the exact threshold among them (two
+//      more radix levels, 11 and 10 bits), the number of rows equal to it
+//      still needed, and from these every warp's output offset and share of
+//      the equal rows, and sends each warp its plan. If some CTA has more
+//      members than CTA 0 has room for, every level is instead a full pass
+//      over the slices, as in step 2, followed by an exchange of per-CTA
+//      counts.
+//   4. Each warp writes its selected rows from its list: the rows above the
+//      threshold and, in position order, as many rows equal to it as its
+//      share (ballots give each row its place). A warp whose list
+//      overflowed walks its run again, 128 rows at a time.
 #include <stdint.h>
 
 #include "common.cuh"

@@ -458,3 +458,36 @@ def test_reuse_rejects_bad_maps():
     assert e.value.status == 1
     assert cache.lens() == [64]
     cache.close()
+
+
+def test_anchor_selection_splits_ties_at_the_threshold():
+    """60 copies of one dominant key at random positions, top_k 30: the
+    threshold is the copies' shared importance and exactly the 30 lowest
+    copies are kept. The copies are few enough for the selection's fast
+    path (their bucket's members go to one CTA) and spread over several
+    CTAs and warps, which split the tied rows in position order."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, top_k = 1, 8, 2, 128, 50000, 4, 64, 30
+    labels = [0, 1]
+    g = Hq // Hkv
+    wl = Workload("split", B, Hq, Hkv, D, T, 1, S, W, 1, seed=15)
+    dq, dk, dv = decode_inputs(wl, 0, device="cuda")
+    k = randn_bf16((B, T, Hkv, D), 151, "cuda")
+    v = randn_bf16((B, T, Hkv, D), 152, "cuda")
+    # a key along the group's summed query direction scores far above the rest
+    qs = dq[0, :g].float().sum(0)
+    k0 = (qs / qs.norm() * 40.0).to(torch.bfloat16)
+    gen = torch.Generator().manual_seed(16)
+    copies = torch.randperm(T, generator=gen)[:60].sort().values
+    k[0, copies.to("cuda"), 0] = k0
+    cache = aoh.Cache(B, Hq, Hkv, D, T + 1, S, W, labels)
+    cache.prefill(None, k, v, None)
+    idx = torch.full((B, 1, top_k), -7, dtype=torch.int32, device="cuda")
+    cache.decode_step_anchor(dq, dk, dv, torch.empty_like(dq), top_k, idx)
+    torch.cuda.synchronize()
+    sel = idx.cpu().numpy()[0, 0]
+    kk = np.concatenate([f64(k[0]), f64(dk[0])[None]])
+    imp = ohs.group_importance(f64(dq[0])[:g], kk[:, 0])
+    _check_selection(sel, imp, top_k)
+    assert np.array_equal(sel, copies.numpy()[:top_k]), (sel, copies.numpy()[:top_k])
+    cache.close()
