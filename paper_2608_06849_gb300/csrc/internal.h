@@ -159,7 +159,7 @@ bool decode_uses_tc(int D, int G);
 // Work units of one gathered row in the reuse step's split on the tcgen05
 // kernel (a 256-byte row gather against a contiguous row's share of a tile
 // stream; measured).
-constexpr int kGatherWeight = 4;
+constexpr int kGatherWeight = 5;
 int decode_tc_ctas(long long total_rows, int num_sms);
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
