@@ -677,10 +677,12 @@ bool make_gather_map(CUtensorMap* tcg, const CacheGeom& g, const void* kv) {
 }
 
 // One CTA per SM; small steps use fewer, at least 512 rows each.
+// At least 512 rows (four tiles) per CTA, so that small steps keep few
+// partials per item (an item spread over more than kGroup CTAs needs the
+// second merge level); once that fills half the GPU, every SM streams.
 int decode_tc_ctas(long long total_rows, int num_sms) {
   const long long by_rows = (total_rows + 511) / 512;
-  long long p = num_sms;
-  if (by_rows < p) p = by_rows;
+  long long p = by_rows >= num_sms / 2 ? num_sms : by_rows;
   return p < 1 ? 1 : (int)p;
 }
 
