@@ -15,7 +15,7 @@ Stage"; Appendix "GQA Extension"):
     head axis (the concatenation of Eq. 8; the W_O projection is not part of
     attention and is not modelled).
 
-Readings taken where the paper is silent (each one is listed in the design doc):
+Readings taken where the paper is silent:
   * the recent window counts the query's own position, so a streaming query
     at position i sees key j iff ``j <= i and (j < S or i - j < W)``;
   * prefill uses that per-token rule for every row by default, which makes

@@ -19,7 +19,7 @@ What the paper fixes:
   * with GQA, similarities of the group pairs are the mean over their query
     head pairs, and all query heads of a group borrow one index set.
 
-Readings taken where the paper is silent (listed in the design doc):
+Readings taken where the paper is silent:
   * the importance of key j for an anchor retrieval group is the sum over
     the group's query heads of their attention probabilities at j (the
     softmax over all positions the head attends); the group keeps the
