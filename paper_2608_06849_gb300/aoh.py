@@ -278,8 +278,19 @@ def aoh_cache_destroy(cache):
 
 # ------------------------------------------------------------- convenience
 
+def _need(t, name, n):
+    """The kernels read or write the first ``n`` elements behind a pointer;
+    a smaller tensor would send them past its end, so it is refused here
+    (the C ABI receives bare pointers and cannot check sizes)."""
+    if t is not None and t.numel() < n:
+        raise ValueError(f"{name} holds {t.numel()} elements; this call needs {n}")
+
+
 class Cache:
-    """A KV buffer on the current CUDA device plus its library handle."""
+    """A KV buffer on the current CUDA device plus its library handle.
+
+    Its methods check every tensor's element count against the cache's
+    configuration before calling the library."""
 
     def __init__(self, batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, labels, device=None, chunk=0):
         self.cfg = make_config(batch, n_q_heads, n_kv_heads, d_head, max_seq, sink, window, chunk)
@@ -290,16 +301,42 @@ class Cache:
         self.batch, self.n_q_heads, self.n_kv_heads, self.d_head = batch, n_q_heads, n_kv_heads, d_head
         self.max_seq, self.sink, self.window, self.chunk = max_seq, sink, window, chunk
 
+    def _check_step(self, q, k_new, v_new, out):
+        nq = self.batch * self.n_q_heads * self.d_head
+        nkv = self.batch * self.n_kv_heads * self.d_head
+        for t, name, n in ((q, "q", nq), (k_new, "k_new", nkv), (v_new, "v_new", nkv), (out, "out", nq)):
+            _need(t, name, n)
+
     def prefill(self, q, k, v, out=None, seq_lens=None, stream=None):
-        aoh_prefill(q, k, v, k.shape[1], seq_lens, self.handle, out, stream)
+        """q, out [B, T, Hq, d] (both may be None: append only); k, v [B, T, Hkv, d]."""
+        T = k.shape[1]
+        nq = self.batch * T * self.n_q_heads * self.d_head
+        nkv = self.batch * T * self.n_kv_heads * self.d_head
+        for t, name, n in ((q, "q", nq), (k, "k", nkv), (v, "v", nkv), (out, "out", nq)):
+            _need(t, name, n)
+        if seq_lens is not None and len(seq_lens) != self.batch:
+            raise ValueError(f"seq_lens has {len(seq_lens)} entries; the cache holds {self.batch} sequences")
+        aoh_prefill(q, k, v, T, seq_lens, self.handle, out, stream)
 
     def decode_step(self, q, k_new, v_new, out, stream=None):
+        """q, out [B, Hq, d]; k_new, v_new [B, Hkv, d]."""
+        self._check_step(q, k_new, v_new, out)
         aoh_decode_step(q, k_new, v_new, self.handle, out, stream)
 
     def decode_step_anchor(self, q, k_new, v_new, out, top_k, indices, stream=None):
+        """As decode_step; indices [B, n_retrieval, top_k] receives the selection."""
+        self._check_step(q, k_new, v_new, out)
+        n_r = sum(1 for x in self.labels if x == RETRIEVAL)
+        _need(indices, "indices", self.batch * n_r * max(0, int(top_k)))
         aoh_decode_step_anchor(q, k_new, v_new, self.handle, out, top_k, indices, stream)
 
     def decode_step_reuse(self, q, k_new, v_new, out, indices, top_k, group_map, stream=None):
+        """As decode_step; indices [B, n_anchor_groups, top_k] from an anchor step."""
+        self._check_step(q, k_new, v_new, out)
+        if indices is not None:
+            if indices.dim() != 3 or indices.shape[0] != self.batch:
+                raise ValueError("indices must be [batch, n_anchor_groups, top_k]")
+            _need(indices, "indices", self.batch * int(indices.shape[1]) * max(0, int(top_k)))
         aoh_decode_step_reuse(q, k_new, v_new, self.handle, out, indices, top_k, group_map, stream)
 
     def lens(self):

@@ -1,0 +1,72 @@
+"""The Python binding refuses tensors too small for the cache's configuration
+before any pointer reaches the library (the C ABI gets bare pointers and
+cannot check sizes). Runs on the CPU: a Cache object is assembled without a
+device buffer, and correctly sized CPU tensors get past the size checks only
+to be refused as non-CUDA tensors."""
+
+import pytest
+import torch
+
+from paper_2608_06849_gb300 import aoh
+
+
+def _cache(B=2, Hq=8, Hkv=2, D=64, labels=(0, 1)):
+    c = object.__new__(aoh.Cache)
+    c.batch, c.n_q_heads, c.n_kv_heads, c.d_head = B, Hq, Hkv, D
+    c.labels = list(labels)
+    c.handle = None
+    return c
+
+
+def _bf16(*shape):
+    return torch.zeros(*shape, dtype=torch.bfloat16)
+
+
+def _needs_cuda(excinfo):
+    return "CUDA tensor" in str(excinfo.value)
+
+
+def test_prefill_sizes():
+    c = _cache()
+    q, kv = _bf16(2, 10, 8, 64), _bf16(2, 10, 2, 64)
+    with pytest.raises(ValueError) as e:
+        c.prefill(q, kv, kv, _bf16(2, 10, 8, 64))
+    assert _needs_cuda(e)
+    for args, name in (((_bf16(2, 9, 8, 64), kv, kv, None), "q"),
+                       ((q, kv, _bf16(2, 10, 1, 64), None), "v"),
+                       ((q, kv, kv, _bf16(1, 10, 8, 64)), "out"),
+                       ((None, _bf16(1, 10, 2, 64), kv, None), "k")):
+        with pytest.raises(ValueError, match=f"^{name} holds"):
+            c.prefill(*args)
+    with pytest.raises(ValueError, match="seq_lens"):
+        c.prefill(q, kv, kv, None, seq_lens=[10])
+
+
+def test_decode_sizes():
+    c = _cache()
+    q, kv = _bf16(2, 8, 64), _bf16(2, 2, 64)
+    with pytest.raises(ValueError) as e:
+        c.decode_step(q, kv, kv, _bf16(2, 8, 64))
+    assert _needs_cuda(e)
+    with pytest.raises(ValueError, match="^out holds"):
+        c.decode_step(q, kv, kv, _bf16(2, 7, 64))
+    with pytest.raises(ValueError, match="^k_new holds"):
+        c.decode_step(q, _bf16(2, 1, 64), kv, q)
+
+
+def test_h2share_index_sizes():
+    c = _cache(labels=(0, 0))
+    q, kv = _bf16(2, 8, 64), _bf16(2, 2, 64)
+    idx = torch.zeros(2, 2, 16, dtype=torch.int32)
+    with pytest.raises(ValueError) as e:
+        c.decode_step_anchor(q, kv, kv, q, 16, idx)
+    assert _needs_cuda(e)
+    with pytest.raises(ValueError, match="^indices holds"):
+        c.decode_step_anchor(q, kv, kv, q, 17, idx)
+    with pytest.raises(ValueError, match="^indices holds"):
+        c.decode_step_reuse(q, kv, kv, q, idx, 17, [0, 1])
+    with pytest.raises(ValueError, match="batch, n_anchor_groups, top_k"):
+        c.decode_step_reuse(q, kv, kv, q, idx.view(4, 16), 16, [0, 1])
+    with pytest.raises(ValueError) as e:
+        c.decode_step_reuse(q, kv, kv, q, idx, 16, [0, 1])
+    assert _needs_cuda(e)
