@@ -70,3 +70,14 @@ def test_h2share_index_sizes():
     with pytest.raises(ValueError) as e:
         c.decode_step_reuse(q, kv, kv, q, idx, 16, [0, 1])
     assert _needs_cuda(e)
+
+
+def test_reuse_group_map_slots():
+    # anchor retrieval groups 1 and 3 hold index-list slots 0 and 1
+    anchor = [1, 0, 1, 0]
+    reuse = [0, 1, 0, 0]
+    head_map = [3, -1, 1, 3]
+    assert aoh.reuse_group_map(head_map, anchor, reuse) == [1, 0, 1]
+    assert aoh.reuse_group_map([0, 0], [1, 1], [1, 1]) == []
+    with pytest.raises(ValueError, match="not an anchor retrieval group"):
+        aoh.reuse_group_map([0, 1, 1, 3], anchor, reuse)
