@@ -81,3 +81,13 @@ def test_reuse_group_map_slots():
     assert aoh.reuse_group_map([0, 0], [1, 1], [1, 1]) == []
     with pytest.raises(ValueError, match="not an anchor retrieval group"):
         aoh.reuse_group_map([0, 1, 1, 3], anchor, reuse)
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """No fallback: without the built library every call raises."""
+    monkeypatch.setattr(aoh, "_lib", None)
+    monkeypatch.setattr(aoh, "LIB_PATH", str(tmp_path / "libaoh.so"))
+    with pytest.raises(RuntimeError, match="is missing"):
+        aoh.aoh_version()
+    with pytest.raises(RuntimeError, match="is missing"):
+        aoh.aoh_cache_bytes(aoh.make_config(1, 8, 2, 64, 16, 2, 4), [0, 1])
