@@ -34,7 +34,8 @@
  * Ownership: the caller allocates and frees the KV buffer, the inputs and the
  * outputs. The handle owns only host state and a small device metadata block
  * (sequence lengths, split-KV scratch, an error word), allocated by
- * aoh_cache_init and released by aoh_cache_destroy.
+ * aoh_cache_init, plus two arrays allocated on first use (the prefill work
+ * list, the H2Share anchor workspace); aoh_cache_destroy releases all of it.
  */
 #ifndef AOH_H_
 #define AOH_H_
@@ -131,6 +132,10 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
  *             or past seq_lens[b] are ignored: their contents (even NaN) do
  *             not affect any output, and their outputs are not written.
  *   out  [B][T][n_q_heads][d_head], or NULL to only fill the cache.
+ * With out, the host lists the call's query tiles (longest first) and uploads
+ * the list to a device array of the handle; the array grows with cudaMalloc
+ * (which synchronises the device) when a call has more tiles than any
+ * earlier call, and aoh_cache_destroy frees it.
  * Errors: INVALID, CAPACITY (a retrieval head would pass max_seq; nothing is
  * launched), CUDA.
  */
