@@ -218,6 +218,12 @@ def aoh_h2share_map(w_q_anchor, w_k_anchor, w_q_reuse, w_k_reuse, anchor_labels,
     anchor-major group similarities."""
     Hq, dh, dm = w_q_anchor.shape
     Hkv = w_k_anchor.shape[0]
+    for t, name, shape in ((w_k_anchor, "w_k_anchor", (Hkv, dh, dm)), (w_q_reuse, "w_q_reuse", (Hq, dh, dm)),
+                           (w_k_reuse, "w_k_reuse", (Hkv, dh, dm))):
+        if tuple(t.shape) != shape:
+            raise ValueError(f"{name} has shape {tuple(t.shape)}; expected {shape}")
+    if len(anchor_labels) != Hkv or len(reuse_labels) != Hkv:
+        raise ValueError(f"anchor_labels and reuse_labels need {Hkv} entries (one per KV head)")
     mp = (ctypes.c_int32 * Hkv)()
     sim = (ctypes.c_double * (Hkv * Hkv))()
     _check(load().aoh_h2share_map(_ptr(w_q_anchor, "w_q_anchor"), _ptr(w_k_anchor, "w_k_anchor"),

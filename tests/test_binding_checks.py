@@ -91,3 +91,16 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
         aoh.aoh_version()
     with pytest.raises(RuntimeError, match="is missing"):
         aoh.aoh_cache_bytes(aoh.make_config(1, 8, 2, 64, 16, 2, 4), [0, 1])
+
+
+def test_h2share_map_shapes():
+    wq, wk = _bf16(8, 64, 96), _bf16(2, 64, 96)
+    with pytest.raises(ValueError, match="^w_q_reuse has shape"):
+        aoh.aoh_h2share_map(wq, wk, _bf16(8, 64, 95), wk, [0, 0], [0, 0])
+    with pytest.raises(ValueError, match="^w_k_anchor has shape"):
+        aoh.aoh_h2share_map(wq, _bf16(2, 64, 95), wq, _bf16(2, 64, 95), [0, 0], [0, 0])
+    with pytest.raises(ValueError, match="entries"):
+        aoh.aoh_h2share_map(wq, wk, wq, wk, [0, 0, 0], [0, 0])
+    with pytest.raises(ValueError) as e:
+        aoh.aoh_h2share_map(wq, wk, wq, wk, [0, 0], [0, 0])
+    assert _needs_cuda(e)
