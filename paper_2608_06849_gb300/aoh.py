@@ -182,6 +182,15 @@ def aoh_decode_step_reuse(q, k_new, v_new, cache, out, indices, top_k, group_map
 def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream=None):
     """The allocation-free decode step: ``kv_buffer`` (CUDA uint8) and ``lens``
     (CUDA int32 [B], advanced by one on the device) belong to the caller."""
+    if len(labels) != cfg.n_kv_heads:
+        raise ValueError(f"labels need {cfg.n_kv_heads} entries (one per KV head)")
+    n_s = sum(1 for x in labels if int(x) == STREAMING)
+    n_r = len(labels) - n_s
+    _need(kv_buffer, "kv_buffer", cfg.batch * (n_r * cfg.max_seq + n_s * (cfg.sink + cfg.window)) * cfg.d_head * 4)
+    _need(lens, "lens", cfg.batch)
+    nq, nkv = cfg.batch * cfg.n_q_heads * cfg.d_head, cfg.batch * cfg.n_kv_heads * cfg.d_head
+    for t, name, n in ((q, "q", nq), (k_new, "k_new", nkv), (v_new, "v_new", nkv), (out, "out", nq)):
+        _need(t, name, n)
     if not lens.is_cuda or lens.dtype != torch.int32 or not lens.is_contiguous():
         raise ValueError("lens must be a contiguous int32 CUDA tensor")
     _check(load().aoh_decode_step_noalloc(

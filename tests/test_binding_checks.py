@@ -104,3 +104,22 @@ def test_h2share_map_shapes():
     with pytest.raises(ValueError) as e:
         aoh.aoh_h2share_map(wq, wk, wq, wk, [0, 0], [0, 0])
     assert _needs_cuda(e)
+
+
+def test_noalloc_sizes():
+    cfg = aoh.make_config(2, 8, 2, 64, 100, 4, 16)
+    labels = [0, 1]
+    kv_bytes = 2 * (100 + 20) * 64 * 4
+    kv = torch.zeros(kv_bytes, dtype=torch.uint8)
+    lens = torch.zeros(2, dtype=torch.int32)
+    q, k1 = _bf16(2, 8, 64), _bf16(2, 2, 64)
+    with pytest.raises(ValueError, match="^kv_buffer holds"):
+        aoh.aoh_decode_step_noalloc(cfg, labels, kv[:-1], lens, 10, q, k1, k1, q)
+    with pytest.raises(ValueError, match="^lens holds"):
+        aoh.aoh_decode_step_noalloc(cfg, labels, kv, lens[:1], 10, q, k1, k1, q)
+    with pytest.raises(ValueError, match="^v_new holds"):
+        aoh.aoh_decode_step_noalloc(cfg, labels, kv, lens, 10, q, k1, k1[:1], q)
+    with pytest.raises(ValueError, match="entries"):
+        aoh.aoh_decode_step_noalloc(cfg, [0], kv, lens, 10, q, k1, k1, q)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        aoh.aoh_decode_step_noalloc(cfg, labels, kv, lens, 10, q, k1, k1, q)
