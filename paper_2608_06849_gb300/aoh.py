@@ -6,7 +6,10 @@ passed as raw device pointers plus the current CUDA stream. There is no
 fallback: if the library is missing or fails to load, every call raises.
 
 ``Cache`` is a small convenience owner of a KV buffer (a torch uint8 device
-tensor) and its handle.
+tensor) and its handle. Its methods, ``aoh_decode_step_noalloc``,
+``aoh_classify`` and ``aoh_h2share_map`` check tensor sizes against the
+configuration; the handle-level functions (``aoh_prefill``,
+``aoh_decode_step`` ...) pass the pointers on unchecked, as the C ABI does.
 """
 
 import ctypes
