@@ -160,3 +160,21 @@ def test_null_handle_calls_fail_cleanly(lib):
     assert lib.aoh_decode_step(None, None, None, None, None, None) == 1
     assert lib.aoh_cache_check(None, None) == 1
     lib.aoh_cache_destroy(None)
+
+
+def test_every_export_has_a_ctypes_signature(lib):
+    """A function without argtypes would have its pointer arguments passed as
+    C ints (truncated on a 64-bit host)."""
+    for name in aoh.EXPORTS:
+        fn = getattr(lib, name)
+        assert fn.argtypes is not None, name
+
+
+def test_ctypes_signatures_match_the_header_arity(lib):
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    decls = dict(re.findall(r"\b(aoh_[a-z0-9_]+)\s*\(([^;{]*?)\)\s*;", text))
+    assert sorted(decls) == sorted(aoh.EXPORTS)
+    for name, params in decls.items():
+        params = " ".join(params.split())
+        n = 0 if params in ("", "void") else params.count(",") + 1
+        assert len(getattr(lib, name).argtypes) == n, (name, params)
