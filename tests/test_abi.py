@@ -178,3 +178,20 @@ def test_ctypes_signatures_match_the_header_arity(lib):
         params = " ".join(params.split())
         n = 0 if params in ("", "void") else params.count(",") + 1
         assert len(getattr(lib, name).argtypes) == n, (name, params)
+
+
+def test_ctypes_argument_types_match_the_header(lib):
+    """Pointers are passed as pointers and integers at their declared width."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    decls = dict(re.findall(r"\b(aoh_[a-z0-9_]+)\s*\(([^;{]*?)\)\s*;", text))
+    scalars = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "size_t": ctypes.c_size_t}
+    for name, params in decls.items():
+        params = " ".join(params.split())
+        if params in ("", "void"):
+            continue
+        for decl, t in zip(params.split(","), getattr(lib, name).argtypes):
+            if "*" in decl:
+                assert t is ctypes.c_void_p or issubclass(t, ctypes._Pointer), (name, decl, t)
+            else:
+                base = [k for k in scalars if re.search(rf"\b{k}\b", decl)]
+                assert base and t is scalars[base[0]], (name, decl, t)
