@@ -195,3 +195,14 @@ def test_ctypes_argument_types_match_the_header(lib):
             else:
                 base = [k for k in scalars if re.search(rf"\b{k}\b", decl)]
                 assert base and t is scalars[base[0]], (name, decl, t)
+
+
+def test_ctypes_return_types_match_the_header(lib):
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    rets = dict((n, r.strip()) for r, n in re.findall(r"(?m)^([A-Za-z_][A-Za-z0-9_ ]*\**)\s*\b(aoh_[a-z0-9_]+)\s*\(",
+                                                    text))
+    assert sorted(rets) == sorted(aoh.EXPORTS)
+    want = {"aoh_status": ctypes.c_int32, "int32_t": ctypes.c_int32, "size_t": ctypes.c_size_t,
+            "const char*": ctypes.c_char_p, "void": None}
+    for name, ret in rets.items():
+        assert getattr(lib, name).restype is want[ret], (name, ret)
