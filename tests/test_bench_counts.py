@@ -40,3 +40,23 @@ def test_reuse_bytes_reduce_to_decode_bytes():
     assert big == bench.decode_bytes(lens, labels, wl) + 4 * n_r * sum(t + 1 for t in lens)
     small = bench.reuse_bytes(lens, labels, wl, 8)
     assert small < big
+
+
+@pytest.mark.parametrize("lens,S,W", [([0, 5, 40], 2, 8), ([100], 0, 1), ([3, 300], 16, 300)])
+def test_decode_bytes_from_the_oracle_mask(lens, S, W):
+    """Bytes of one decode step counted from the keys the oracle lets the new
+    token see: every visible cached row read once (K and V), the new token's
+    K/V read and appended, q read and out written."""
+    import dataclasses
+
+    from paper_2608_06849_gb300.workloads import DECODE_128K
+    wl = dataclasses.replace(DECODE_128K, batch=len(lens), sink=S, window=W)
+    labels = [0, 1, 1, 0, 1, 0, 0, 1]
+    row = wl.d_head * 2
+    want = 0
+    for t in lens:
+        for lab in labels:
+            seen = int(oatt.allowed_mask(np.array([t]), np.arange(t + 1), lab == 1, S, W).sum())
+            want += (seen - 1) * row * 2 + row * 2 * 2
+        want += wl.n_q_heads * wl.d_head * 2 * 2
+    assert bench.decode_bytes(lens, labels, wl) == want
