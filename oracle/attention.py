@@ -2,7 +2,8 @@
 
 TEST INFRASTRUCTURE ONLY (see the package docstring): the plain float64
 definition that the CUDA path is compared with. Parity status: pinned
-(brute force, closed forms, a library attention routine, invariants) by
+(brute force, closed forms, a library attention routine, invariants, and
+both forms of the mask against the rule written out pair by pair) by
 ``tests/test_oracle_attention.py``.
 
 What the paper fixes (Sec. 5, "Decode Stage", Eq. 8 and "Chunked-Prefill

@@ -12,7 +12,9 @@ the module disagrees with what the paper and the mathematics fix:
   * the chunk-eviction option against a step-by-step simulation of the
     procedure of the "Chunked-Prefill Stage" (process a chunk against the
     cache, then evict all but the sinks and the W most recent tokens), plus
-    two closed forms (chunks of one token; one chunk covering the prompt).
+    two closed forms (chunks of one token; one chunk covering the prompt);
+  * the scalar and the vector form of the mask against the mask conditions
+    written out here, over every (query, key) pair of small cases.
 """
 
 import math
@@ -250,6 +252,41 @@ def pin_chunk_closed_forms(att):
     np.testing.assert_array_equal(att.prefill(q, k, v, [1, 0], 2, 4, chunk=0), att.prefill(q, k, v, [1, 0], 2, 4))
 
 
+def _mask_written_out(i, j, streaming, S, W, chunk):
+    """The visibility rule as Sec. 5 states it, with the readings of the
+    module docstring: causal; a streaming head keeps the S sinks and either
+    the W positions up to the query (per-token window) or, with eviction
+    after each chunk of K tokens, the W positions before the query's chunk
+    plus the chunk itself."""
+    if j > i:
+        return False
+    if not streaming or j < S:
+        return True
+    if chunk == 0:
+        return j > i - W
+    chunk_start = i - i % chunk
+    return j >= chunk_start - W
+
+
+def pin_scalar_mask(att):
+    """``allowed`` (scalar) and ``allowed_mask`` (vector) over every pair
+    (i, j) of small cases, with and without the chunk rule, against the
+    conditions written out above."""
+    for streaming in (False, True):
+        for S in (0, 1, 3):
+            for W in (1, 2, 5):
+                for chunk in (0, 1, 3, 4):
+                    T = 3 * (S + W) + 2 * max(chunk, 1) + 1
+                    mask = att.allowed_mask(np.arange(T), np.arange(T), streaming, S, W, chunk)
+                    assert mask.shape == (T, T)
+                    for i in range(T):
+                        for j in range(T):
+                            want = _mask_written_out(i, j, streaming, S, W, chunk)
+                            assert bool(att.allowed(i, j, streaming, S, W, chunk)) == want, (
+                                "allowed", i, j, streaming, S, W, chunk)
+                            assert bool(mask[i, j]) == want, ("allowed_mask", i, j, streaming, S, W, chunk)
+
+
 ALL_PINS = [
     pin_brute_force,
     pin_library_sdpa,
@@ -261,4 +298,5 @@ ALL_PINS = [
     pin_ring_slot_layout,
     pin_chunk_eviction_simulation,
     pin_chunk_closed_forms,
+    pin_scalar_mask,
 ]

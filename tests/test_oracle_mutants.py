@@ -31,6 +31,10 @@ MUTANTS = {
     "chunk_window_off_by_one": ("(j >= (i // chunk) * chunk - W))", "(j > (i // chunk) * chunk - W))"),
     "chunk_per_query": ("(j >= (i // chunk) * chunk - W))", "(j >= i - W))"),
     "chunk_ignored": ("    if chunk:\n        return causal", "    if False:\n        return causal"),
+    # the scalar form alone (the vector form, which prefill uses, untouched)
+    "scalar_window_off_by_one": ("return j < S or i - j < W", "return j < S or i - j <= W"),
+    "scalar_chunk_per_query": ("return j < S or j >= (i // chunk) * chunk - W", "return j < S or j >= i - W"),
+    "scalar_not_causal": ("    if j > i:\n        return False", "    if j > i + 1:\n        return False"),
 }
 
 
