@@ -32,10 +32,11 @@
  *     arguments are caught on the host before anything is launched.
  *
  * Ownership: the caller allocates and frees the KV buffer, the inputs and the
- * outputs. The handle owns only host state and a small device metadata block
- * (sequence lengths, split-KV scratch, an error word), allocated by
- * aoh_cache_init, plus two arrays allocated on first use (the prefill work
- * list, the H2Share anchor workspace); aoh_cache_destroy releases all of it.
+ * outputs. The handle owns only host state and device arrays it allocates
+ * itself: a small metadata block (sequence lengths, split-KV scratch, an
+ * error word) and the prefill work list, both allocated by aoh_cache_init,
+ * and the H2Share anchor workspace, allocated by aoh_cache_reserve or on the
+ * first anchor step; aoh_cache_destroy releases all of it.
  */
 #ifndef AOH_H_
 #define AOH_H_
@@ -107,8 +108,10 @@ size_t aoh_cache_bytes(const aoh_config* cfg, const uint8_t* head_labels);
  * stores position p < S at row p and position p >= S at row
  * S + (p - S) mod W (a ring of W rows after the sinks). aoh_cache_region()
  * returns the offsets.
- * Synchronises the device once (metadata upload). Errors: INVALID, CAPACITY,
- * UNSUPPORTED, CUDA.
+ * Allocates the handle's metadata block and a prefill work list sized for
+ * chunks of up to max_seq tokens (B * n_q_heads * ceil(max_seq / 256)
+ * entries of 16 bytes), and synchronises the device once (metadata upload).
+ * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
                           size_t kv_buffer_bytes, aoh_cache** out);
@@ -133,9 +136,10 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
  *             not affect any output, and their outputs are not written.
  *   out  [B][T][n_q_heads][d_head], or NULL to only fill the cache.
  * With out, the host lists the call's query tiles (longest first) and uploads
- * the list to a device array of the handle; the array grows with cudaMalloc
- * (which synchronises the device) when a call has more tiles than any
- * earlier call, and aoh_cache_destroy frees it.
+ * the list to the handle's work list. A chunk of at most max_seq tokens (or
+ * of at most the max_tokens given to aoh_cache_reserve) fits the list as
+ * allocated; only a longer chunk, which a cache without retrieval heads can
+ * take, grows it with cudaMalloc (which synchronises the device).
  * Errors: INVALID, CAPACITY (a retrieval head would pass max_seq; nothing is
  * launched), CUDA.
  */
@@ -169,9 +173,10 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
  *   indices  device int32 [B][n_r][top_k] (n_r = retrieval KV heads, in
  *            increasing KV-head index), written on the stream; entries past
  *            min(top_k, t + 1) are -1.
- * Needs d_head 128 (the tensor-core decode). The first call allocates a
- * workspace of about B * n_r * max_seq * (group size) floats in the handle,
- * plus B * n_r * max_seq more when max_seq exceeds 147456 (a cudaMalloc,
+ * Needs d_head 128 (the tensor-core decode). Uses a workspace of about
+ * B * n_r * max_seq * (group size) floats in the handle, plus
+ * B * n_r * max_seq more when max_seq exceeds 147456; aoh_cache_reserve
+ * allocates it up front, else the first anchor step does (a cudaMalloc,
  * which synchronises the device); aoh_cache_destroy frees it.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
@@ -237,6 +242,19 @@ aoh_status aoh_h2share_map(const void* w_q_anchor, const void* w_k_anchor, const
                            int32_t d_model, const uint8_t* anchor_labels, const uint8_t* reuse_labels,
                            int32_t* map_out, double* group_sim_out, void* stream);
 
+/*
+ * Allocate now the device arrays that later calls would otherwise allocate on
+ * first use (the paper has no counterpart): the prefill work list for chunks
+ * of up to max_tokens tokens (aoh_cache_init already sized it for max_seq),
+ * and, if anchor_workspace is nonzero, the H2Share anchor workspace of
+ * aoh_decode_step_anchor. A caller that must not allocate while serving calls
+ * this once after aoh_cache_init; calls within these limits then allocate
+ * nothing. Uses cudaMalloc (which synchronises the device) for what is not
+ * yet allocated. Errors: INVALID, UNSUPPORTED (anchor workspace without the
+ * d_head 128 tensor-core decode), CUDA.
+ */
+aoh_status aoh_cache_reserve(aoh_cache* cache, int32_t max_tokens, int32_t anchor_workspace);
+
 /* Copy the host-side lengths (tokens held per sequence) into lens_out [B]. */
 aoh_status aoh_cache_lens(const aoh_cache* cache, int32_t* lens_out);
 
@@ -252,8 +270,10 @@ aoh_status aoh_cache_reset(aoh_cache* cache, void* stream);
 
 /*
  * Synchronise `stream` and read the device error word that kernels set when
- * a bounded wait runs out. Returns AOH_OK, AOH_ERR_TIMEOUT (and clears the
- * word) or AOH_ERR_CUDA.
+ * a bounded wait runs out (or when a decode step finds a sequence already
+ * holding max_seq tokens, which the host checks prevent on this handle).
+ * Returns AOH_OK, AOH_ERR_TIMEOUT or AOH_ERR_CAPACITY (and clears the word),
+ * or AOH_ERR_CUDA.
  */
 aoh_status aoh_cache_check(aoh_cache* cache, void* stream);
 
@@ -296,8 +316,10 @@ const char* aoh_last_error(void);
  *   lens       device int32 [B]: tokens held per sequence before the step;
  *              each entry is advanced by one on the device.
  *   max_len    host upper bound of every lens[b]; used for the split schedule
- *              and the capacity check (max_len + 1 <= max_seq when a
- *              retrieval head exists).
+ *              and the host capacity check (max_len + 1 <= max_seq when a
+ *              retrieval head exists). A bound that is too low (e.g. a
+ *              CUDA graph captured once and replayed for many steps) still
+ *              gives correct outputs, with a less even split.
  *   q, k_new, v_new, out  as for aoh_decode_step.
  *
  * Limits and behaviour:
@@ -312,14 +334,33 @@ const char* aoh_last_error(void);
  *     ends. Calls whose kernels overlap on the GPU (on different streams, or
  *     from different threads without ordering) race on the scratch and
  *     produce wrong results: order them on one stream.
- *   - A bounded-wait timeout inside the kernel is not reported by this call
- *     and leaves the outputs of that call unspecified; the launch still
- *     leaves the scratch clean for the next call.
+ *   - The kernel also checks capacity on the device: a sequence whose
+ *     lens[b] already equals max_seq (with a retrieval head present) is
+ *     skipped: nothing is appended, its outputs are not written and lens[b]
+ *     stays as it is. Such a step, and a bounded-wait timeout inside the
+ *     kernel (whose outputs are then unspecified), are not reported by this
+ *     asynchronous call; they set bits of a sticky status word that
+ *     aoh_decode_step_noalloc_status() reads. Either way the launch leaves
+ *     the scratch clean for the next call.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
                                    int32_t* lens, int32_t max_len, const void* q, const void* k_new,
                                    const void* v_new, void* out, void* stream);
+
+/*
+ * Status of the allocation-free decode steps on the current device since the
+ * last query (the paper has no counterpart). Synchronises `stream` (order
+ * every aoh_decode_step_noalloc call of the device on it, or synchronise
+ * them first), reads the sticky status word kept in the same static array
+ * and clears it; allocates nothing.
+ *   flags  host uint32 (may be NULL): 1 = a bounded wait ran out (those
+ *          outputs are unspecified), 2 = a step found a sequence already
+ *          holding max_seq tokens (that sequence was skipped); 0 if neither.
+ * Returns AOH_OK, AOH_ERR_TIMEOUT (bit 1 set), AOH_ERR_CAPACITY (bit 2
+ * alone) or AOH_ERR_CUDA.
+ */
+aoh_status aoh_decode_step_noalloc_status(uint32_t* flags, void* stream);
 
 /*
  * Effective-rank head classification (Sec. 4, Eq. 2-6 and Algorithm 1;
@@ -351,7 +392,8 @@ aoh_status aoh_classify(const void* w_q, const void* w_k, int32_t n_layers, int3
                         int32_t n_kv_heads, int32_t d_head, int32_t d_model, int32_t sparsity_pct,
                         double* er_out, uint8_t* labels_out, void* stream);
 
-/* Library ABI version (major * 100 + minor); 101 added aoh_config.chunk. */
+/* Library ABI version (major * 100 + minor); 101 added aoh_config.chunk, 102
+ * aoh_cache_reserve and aoh_decode_step_noalloc_status. */
 int32_t aoh_version(void);
 
 #ifdef __cplusplus

@@ -33,11 +33,13 @@ EXPORTS = [
     "aoh_cache_lens",
     "aoh_cache_region",
     "aoh_cache_reset",
+    "aoh_cache_reserve",
     "aoh_cache_check",
     "aoh_cache_destroy",
     "aoh_last_error",
     "aoh_version",
     "aoh_decode_step_noalloc",
+    "aoh_decode_step_noalloc_status",
     "aoh_classify",
     "aoh_decode_step_anchor",
     "aoh_decode_step_reuse",
@@ -84,6 +86,7 @@ def load():
         "aoh_cache_lens": (i32, [P, i32p]),
         "aoh_cache_region": (i32, [P, i32, i32, szp, szp, i32p]),
         "aoh_cache_reset": (i32, [P, P]),
+        "aoh_cache_reserve": (i32, [P, i32, i32]),
         "aoh_cache_check": (i32, [P, P]),
         "aoh_h2share_map": (i32, [P, P, P, P, i32, i32, i32, i32, u8p, u8p, i32p,
                                   ctypes.POINTER(ctypes.c_double), P]),
@@ -92,6 +95,7 @@ def load():
         "aoh_last_error": (ctypes.c_char_p, []),
         "aoh_version": (i32, []),
         "aoh_decode_step_noalloc": (i32, [cfgp, u8p, P, i32p, i32, P, P, P, P, P]),
+        "aoh_decode_step_noalloc_status": (i32, [ctypes.POINTER(ctypes.c_uint32), P]),
         "aoh_classify": (i32, [P, P, i32, i32, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), u8p, P]),
     }
     for name, (res, args) in sig.items():
@@ -202,6 +206,19 @@ def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_n
         _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), _ptr(out, "out"), _stream_ptr(stream)))
 
 
+def aoh_decode_step_noalloc_status(stream=None):
+    """Read and clear the allocation-free decode's sticky status word on the
+    current device (after synchronising ``stream``). Returns
+    ``(status, flags)``: status is AOH_OK, 4 (TIMEOUT) or 2 (CAPACITY);
+    flags holds bit 1 (a bounded wait ran out) and bit 2 (a step found a
+    sequence already holding max_seq tokens). Does not raise on those."""
+    flags = ctypes.c_uint32(0)
+    st = load().aoh_decode_step_noalloc_status(ctypes.byref(flags), _stream_ptr(stream))
+    if st not in (AOH_OK, 2, 4):
+        _check(st)
+    return st, flags.value
+
+
 def aoh_classify(w_q, w_k, n_kv_heads, sparsity_pct, stream=None):
     """Effective-rank labels. w_q [L, Hq, d_head, d_model] and w_k
     [L, Hkv, d_head, d_model] (or one layer without the leading L) are
@@ -277,6 +294,13 @@ def aoh_cache_region(cache, b, kv_head):
 
 def aoh_cache_reset(cache, stream=None):
     _check(load().aoh_cache_reset(cache, _stream_ptr(stream)))
+
+
+def aoh_cache_reserve(cache, max_tokens, anchor_workspace=False):
+    """Allocate the prefill work list for chunks of up to max_tokens tokens
+    and, optionally, the H2Share anchor workspace, so later calls within
+    those limits allocate nothing."""
+    _check(load().aoh_cache_reserve(cache, int(max_tokens), 1 if anchor_workspace else 0))
 
 
 def aoh_cache_check(cache, stream=None):
@@ -370,6 +394,9 @@ class Cache:
 
     def reset(self, stream=None):
         aoh_cache_reset(self.handle, stream)
+
+    def reserve(self, max_tokens, anchor_workspace=False):
+        aoh_cache_reserve(self.handle, max_tokens, anchor_workspace)
 
     def check(self, stream=None):
         aoh_cache_check(self.handle, stream)

@@ -132,9 +132,41 @@ struct aoh_cache {
   float* d_h2 = nullptr;
 };
 
+namespace {
+
+// Grow the prefill work list to at least n items (cudaMalloc, which
+// synchronises the device).
+cudaError_t reserve_work(aoh_cache* h, size_t n) {
+  if (n <= h->work_cap) return cudaSuccess;
+  if (h->d_work) cudaFree(h->d_work);
+  h->d_work = nullptr;
+  h->work_cap = 0;
+  cudaError_t e = cudaMalloc(&h->d_work, n * sizeof(int4));
+  if (e == cudaSuccess) h->work_cap = n;
+  return e;
+}
+
+// Work items of a prefill call whose chunks hold up to `tokens` rows: one per
+// (sequence, query head, 256-row pair of query tiles).
+size_t work_items_for(const CacheGeom& g, long long tokens) {
+  return (size_t)g.B * g.Hq * (size_t)((tokens + 255) / 256);
+}
+
+// The H2Share anchor workspace (once per handle; cudaMalloc).
+cudaError_t reserve_h2(aoh_cache* h) {
+  const CacheGeom& g = h->geom;
+  if (g.n_r == 0 || h->d_h2) return cudaSuccess;
+  // scores [B][n_r][G][max_seq padded to 4], head states, importance overflow
+  cudaError_t e = cudaMalloc(&h->d_h2, h2_workspace_floats(g.B, g.n_r, g.G, g.max_seq) * sizeof(float));
+  if (e != cudaSuccess) h->d_h2 = nullptr;
+  return e;
+}
+
+}  // namespace
+
 extern "C" {
 
-int32_t aoh_version(void) { return 101; }
+int32_t aoh_version(void) { return 102; }
 
 const char* aoh_last_error(void) { return g_last_error.c_str(); }
 
@@ -224,7 +256,29 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
     delete h;
     return fail(AOH_ERR_CUDA, "cuTensorMapEncodeTiled failed for the cache regions");
   }
+  // the prefill work list for the longest chunk a retrieval head can take
+  // (max_seq tokens), so that prefill calls within it allocate nothing
+  e = reserve_work(h, work_items_for(h->geom, c.max_seq));
+  if (e != cudaSuccess) {
+    cudaFree(h->meta);
+    delete h;
+    return cuda_fail(e, "work list allocation");
+  }
   *out = h;
+  return AOH_OK;
+}
+
+aoh_status aoh_cache_reserve(aoh_cache* cache, int32_t max_tokens, int32_t anchor_workspace) {
+  if (!cache) return fail(AOH_ERR_INVALID, "cache is NULL");
+  if (max_tokens < 0) return fail(AOH_ERR_INVALID, "max_tokens must be >= 0");
+  cudaError_t e = reserve_work(cache, work_items_for(cache->geom, max_tokens));
+  if (e != cudaSuccess) return cuda_fail(e, "work list allocation");
+  if (anchor_workspace) {
+    if (!decode_uses_tc(cache->geom.D, cache->geom.G))
+      return fail(AOH_ERR_UNSUPPORTED, "the anchor step needs the d_head 128 tensor-core decode");
+    e = reserve_h2(cache);
+    if (e != cudaSuccess) return cuda_fail(e, "anchor workspace allocation");
+  }
   return AOH_OK;
 }
 
@@ -272,7 +326,9 @@ aoh_status aoh_cache_check(aoh_cache* cache, void* stream) {
   if (err) {
     const uint32_t zero = 0;
     cudaMemcpy(cache->d_err, &zero, sizeof(zero), cudaMemcpyHostToDevice);
-    return fail(AOH_ERR_TIMEOUT, "a kernel's bounded wait ran out (error word 0x%x)", err);
+    if (err & kErrTimeout) return fail(AOH_ERR_TIMEOUT, "a kernel's bounded wait ran out (error word 0x%x)", err);
+    return fail(AOH_ERR_CAPACITY, "a decode step found a sequence already holding max_seq tokens (error word 0x%x)",
+                err);
   }
   return AOH_OK;
 }
@@ -333,14 +389,8 @@ aoh_status aoh_prefill(const void* q, const void* k, const void* v, int32_t T, c
   if (out) {
     const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)g.D));
     std::vector<int4> items = prefill_schedule(g, base, clen);
-    if (items.size() > cache->work_cap) {
-      if (cache->d_work) cudaFree(cache->d_work);
-      cache->d_work = nullptr;
-      cache->work_cap = 0;
-      e = cudaMalloc(&cache->d_work, items.size() * sizeof(int4));
-      if (e != cudaSuccess) return cuda_fail(e, "work list allocation");
-      cache->work_cap = items.size();
-    }
+    e = reserve_work(cache, items.size());
+    if (e != cudaSuccess) return cuda_fail(e, "work list allocation");
     e = cudaMemcpyAsync(cache->d_work, items.data(), items.size() * sizeof(int4), cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work)");
     PrefillTcArgs pa;
@@ -446,14 +496,8 @@ aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* 
   if (!decode_uses_tc(g.D, g.G))
     return fail(AOH_ERR_UNSUPPORTED, "the anchor step needs the d_head 128 tensor-core decode");
   if (g.n_r > 0 && !cache->d_h2) {
-    // scores [B][n_r][G][max_seq padded to 4], head states, importance overflow
-    const size_t n = h2_workspace_floats(g.B, g.n_r, g.G, g.max_seq);
-    cudaError_t e = cudaMalloc(&cache->d_h2, n * sizeof(float));
-    if (e != cudaSuccess) {
-      if (cache->d_h2) cudaFree(cache->d_h2);
-      cache->d_h2 = nullptr;
-      return cuda_fail(e, "anchor workspace allocation");
-    }
+    cudaError_t e = reserve_h2(cache);
+    if (e != cudaSuccess) return cuda_fail(e, "anchor workspace allocation");
   }
   if (g.n_r > 0) h2_decode_outputs(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, &a.scores, &a.score_stride, &a.score_stats);
   a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);

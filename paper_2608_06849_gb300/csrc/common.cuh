@@ -6,10 +6,11 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "internal.h"
+
 namespace aoh {
 
-// Bits of the device error word.
-constexpr uint32_t kErrTimeout = 1u;
+// Bits of the device error word: kErrTimeout, kErrCapacity (internal.h).
 
 // A bounded wait gives up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;

@@ -27,14 +27,23 @@ __device__ __forceinline__ int seq_len(const DecodeArgs& a, int b, const int* le
   return lens_s ? lens_s[b] : __ldcg(&a.lens[b]);
 }
 
+// A sequence whose retrieval heads are already full (t >= max_seq) cannot
+// take the new token: the step skips every item of it (nothing appended,
+// no output written) and the launch's last CTA leaves its length as it is
+// and flags kErrCapacity. The host checks its mirror of the lengths before
+// a handle launch; this guard covers callers whose host bound can go stale
+// (the allocation-free entry point, e.g. replayed from a CUDA graph).
+__device__ __forceinline__ bool seq_full(const CacheGeom& g, int t) { return g.n_r > 0 && t >= g.max_seq; }
+
 // Rows of item `id`. Retrieval: t + 1 rows (min(top_k, t + 1) borrowed rows
 // in the H2Share reuse step); streaming: min(t + 1, S + W) ring rows;
-// t = tokens held before this step.
+// t = tokens held before this step. 0 for every item of a full sequence.
 __device__ __forceinline__ int item_rows(const DecodeArgs& a, int id, const int* lens_s = nullptr) {
   const CacheGeom& g = a.geom;
   const int HK = g.n_r + g.n_s;
   const int b = id / HK, k = id - b * HK;
   const int t = seq_len(a, b, lens_s);
+  if (seq_full(g, t)) return 0;
   if (k < g.n_r) return a.idx ? min(a.top_k, t + 1) : t + 1;
   return min(t + 1, g.S + g.W);
 }
@@ -327,20 +336,38 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
   merge_parts<G, D, NT, WIDE>(n_groups, grp_part, outp, nullptr, scratch, stats);
 }
 
-// The launch's last CTA advances every sequence length by one. Called by
-// thread 0 after a __syncthreads that follows all of the CTA's work. A
-// completed merge leaves its counters at zero; after a timeout some may be
-// left behind, and a self-cleaning launch zeroes them and the error word.
+// The launch's last CTA advances every sequence length by one, except
+// those of full sequences (seq_full), which it flags with kErrCapacity.
+// Called by thread 0 after a __syncthreads that follows all of the CTA's
+// work. A completed merge leaves its counters at zero; after a timeout some
+// may be left behind, and a self-cleaning launch zeroes them and the error
+// word. The launch's flags (timeout, capacity) are also ORed into the
+// sticky status word when there is one; nothing in a launch clears it.
 __device__ __forceinline__ void finish_launch(const DecodeArgs& a) {
   __threadfence();
   const uint32_t prev = atomicAdd(a.done, 1u);
   if (prev == gridDim.x - 1) {
-    for (int i = 0; i < a.geom.B; ++i) a.lens[i] += 1;
-    if (a.self_clean && *reinterpret_cast<volatile uint32_t*>(a.err) != 0u) {
-      const int items = a.geom.B * (a.geom.n_r + a.geom.n_s);
-      for (int i = 0; i < items; ++i) a.counters[i] = 0u;
-      for (int i = 0; i < 2 * (int)gridDim.x; ++i) a.gcounters[i] = 0u;
-      *a.err = 0u;
+    __threadfence();
+    bool full = false;
+    for (int i = 0; i < a.geom.B; ++i) {
+      const int t = a.lens[i];
+      if (seq_full(a.geom, t))
+        full = true;
+      else
+        a.lens[i] = t + 1;
+    }
+    const uint32_t e = *reinterpret_cast<volatile uint32_t*>(a.err);
+    const uint32_t flags = e | (full ? kErrCapacity : 0u);
+    if (a.status != nullptr && flags != 0u) atomicOr(a.status, flags);
+    if (a.self_clean) {
+      if (e != 0u) {
+        const int items = a.geom.B * (a.geom.n_r + a.geom.n_s);
+        for (int i = 0; i < items; ++i) a.counters[i] = 0u;
+        for (int i = 0; i < 2 * (int)gridDim.x; ++i) a.gcounters[i] = 0u;
+        *a.err = 0u;
+      }
+    } else if (full) {
+      atomicOr(a.err, kErrCapacity);
     }
     __threadfence();
     *a.done = 0u;

@@ -20,12 +20,14 @@
 #include <mutex>
 
 #include "../../include/aoh.h"
+#include "common.cuh"
 #include "internal.h"
 
 namespace aoh {
 namespace {
 
-constexpr size_t kNoAllocHeaderBytes = 128 * 1024;        // err, done, item and group counters
+constexpr size_t kNoAllocHeaderBytes = 128 * 1024;        // err, status, done, item and group counters
+constexpr int kStatusWord = 16;                            // sticky status: header word 16
 constexpr size_t kNoAllocPartialBytes = 16u * 1024 * 1024;  // split-KV partials
 constexpr size_t kNoAllocScratchBytes = kNoAllocHeaderBytes + kNoAllocPartialBytes;
 constexpr int kNoAllocMaxItems = 16320;  // B * n_kv_heads limit
@@ -156,8 +158,31 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
   a.n_ctas = n_ctas;
   a.self_clean = 1;
+  a.status = header + kStatusWord;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));
   e = launch_decode(a, s);
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: kernel launch failed");
   return AOH_OK;
+}
+
+extern "C" aoh_status aoh_decode_step_noalloc_status(uint32_t* flags, void* stream) {
+  if (flags) *flags = 0u;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc_status: cudaStreamSynchronize failed");
+  // read and clear the sticky word of the current device's array (no
+  // allocation: symbol copies into and out of a host variable)
+  uint32_t w = 0u;
+  const size_t at = kStatusWord * sizeof(uint32_t);
+  e = cudaMemcpyFromSymbol(&w, g_noalloc_scratch, sizeof(w), at, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc_status: cudaMemcpyFromSymbol failed");
+  if (w == 0u) return AOH_OK;
+  const uint32_t zero = 0u;
+  e = cudaMemcpyToSymbol(g_noalloc_scratch, &zero, sizeof(zero), at, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc_status: cudaMemcpyToSymbol failed");
+  if (flags) *flags = w;
+  if (w & kErrTimeout)
+    return set_err(AOH_ERR_TIMEOUT, "aoh_decode_step_noalloc: a kernel's bounded wait ran out since the last query");
+  return set_err(AOH_ERR_CAPACITY,
+                 "aoh_decode_step_noalloc: a step found a sequence already holding max_seq tokens since the last query");
 }

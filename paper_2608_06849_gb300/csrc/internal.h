@@ -11,6 +11,11 @@ namespace aoh {
 
 constexpr int kMaxKvHeads = 64;
 
+// Bits of the device error word (and of the allocation-free entry point's
+// sticky status word).
+constexpr uint32_t kErrTimeout = 1u;   // a kernel's bounded wait ran out
+constexpr uint32_t kErrCapacity = 2u;  // a decode step found a sequence already holding max_seq tokens
+
 // Cache geometry as the kernels see it. Offsets are in bf16 elements from the
 // cache base; see include/aoh.h for the layout.
 struct CacheGeom {
@@ -65,6 +70,9 @@ struct DecodeArgs {
   // counter at zero after a timed-out launch, so the next launch needs no
   // clearing (the allocation-free entry point, which reports no timeouts)
   int self_clean = 0;
+  // sticky status (or null): the last CTA ORs in the launch's kErrTimeout /
+  // kErrCapacity flags; only the host clears it (allocation-free entry point)
+  uint32_t* status = nullptr;
   float scale_log2;   // log2(e) / sqrt(D)
   // H2Share anchor step (tcgen05 kernel): when non-null, every retrieval row's
   // scores (log2 units) go to scores[((b * n_r + i) * G + h) * score_stride + row],

@@ -55,7 +55,7 @@ def test_noalloc_rejects_bad_arguments_on_host(lib):
 
 
 def test_version(lib):
-    assert aoh.aoh_version() == 101
+    assert aoh.aoh_version() == 102
 
 
 @pytest.mark.parametrize("B,Hq,Hkv,d,max_seq,S,W,labels", [
