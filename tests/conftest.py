@@ -29,3 +29,19 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+def pytest_sessionfinish(session, exitstatus):
+    """Write the raw parity figures of the full-size checks (max and mean
+    |err| against the oracle) to the file AOH_PARITY_LOG names, if any."""
+    path = os.environ.get("AOH_PARITY_LOG")
+    if not path:
+        return
+    mod = sys.modules.get("gpu_cases")
+    figs = getattr(mod, "FIGURES", None) if mod else None
+    if not figs:
+        return
+    import json
+    with open(path, "w") as f:
+        for name in sorted(figs):
+            f.write(json.dumps(dict(check=name, **figs[name])) + "\n")

@@ -11,6 +11,12 @@ from paper_2608_06849_gb300.workloads import Workload, decode_inputs, prefill_in
 
 MAX_ABS = 1e-2    # the bound on max |err| against the oracle
 MEAN_ABS = 1e-3   # the bound on mean |err|
+RAW_EXEMPT = 2.0  # |o| from which bf16 output rounding (up to 2^-8 there) plus P rounding can pass 1e-2
+
+# raw figures of the full-size checks by name (max and mean |err|, elements,
+# the max over elements with |o| < RAW_EXEMPT, the count over 1e-2, the worst
+# three); written out by conftest.py when AOH_PARITY_LOG names a file
+FIGURES = {}
 
 _built = False
 
@@ -63,6 +69,38 @@ def assert_matches(got, want, what="", mag=None, abs_bounds=True):
     return err.max(), err.mean()
 
 
+def assert_raw(got, want, what):
+    """The plain figures against the oracle, with no allowance for the bf16
+    output format: mean |err| <= 1e-3 always, and max |err| <= 1e-2 for every
+    element with |o| < RAW_EXEMPT. Above that magnitude storing the exact
+    value in bf16 alone costs up to 2^-9 |o| (2^-8 at |o| = 2), and rounding
+    the softmax weights to bf16 before P.V adds up to 2^-9 of the weighted
+    |v| (R4), so a few such elements can pass 1e-2; they are recorded with
+    their |o| (and are held to the bound beyond the output rounding by
+    assert_matches). Records the figures under ``what``."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    err = np.abs(got - want)
+    small = np.abs(want) < RAW_EXEMPT
+    mx_small = float(err[small].max()) if small.any() else 0.0
+    over = err > MAX_ABS
+    worst = [{"abs_err": float(err.flat[i]), "abs_o": float(abs(want.flat[i])),
+              "bf16_floor": float(abs(bf16_round(want.flat[i]) - want.flat[i]))}
+             for i in np.argsort(err, axis=None)[::-1][:3]]
+    prev = FIGURES.get(what)
+    n = err.size + (prev["elements"] if prev else 0)
+    rec = {"max_abs_err": max(float(err.max()), prev["max_abs_err"] if prev else 0.0),
+           "mean_abs_err": (float(err.sum()) + (prev["mean_abs_err"] * prev["elements"] if prev else 0.0)) / n,
+           "elements": n,
+           "max_abs_err_where_abs_o_below_exempt": max(mx_small, prev["max_abs_err_where_abs_o_below_exempt"]
+                                                        if prev else 0.0),
+           "elements_over_1e-2": int(over.sum()) + (prev["elements_over_1e-2"] if prev else 0),
+           "worst": sorted((prev["worst"] if prev else []) + worst, key=lambda w: -w["abs_err"])[:3]}
+    FIGURES[what] = rec
+    assert mx_small <= MAX_ABS, f"{what}: raw max |err| {mx_small:.3e} where |o| < {RAW_EXEMPT}; worst {worst}"
+    assert err.mean() <= MEAN_ABS, f"{what}: raw mean |err| {err.mean():.3e}"
+
+
 def check_cache_image(cache, k, v, lens, labels, S, W):
     """Bit-exact: retrieval rows 0..len-1 hold K/V of positions 0..len-1;
     streaming rows hold the sink and ring image the oracle's slot model gives."""
@@ -84,7 +122,7 @@ def check_cache_image(cache, k, v, lens, labels, S, W):
 
 
 def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink_scale=8.0, seed=0,
-             check_prefill_out=True, peaky=1.0, rows=None, abs_bounds=True):
+             check_prefill_out=True, peaky=1.0, rows=None, abs_bounds=True, raw_name=None):
     """Prefill (+ decode steps) on the GPU; every output compared with the oracle."""
     ensure_lib()
     wl = Workload("case", B, Hq, Hkv, d, T, decode_steps, S, W, sum(labels), seed=seed, sink_scale=sink_scale)
@@ -106,6 +144,8 @@ def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink
             want = oatt.prefill(qn[b, :lens[b]], kn[b, :lens[b]], vn[b, :lens[b]], labels, S, W, rows=r)
             mag = oatt.prefill(qn[b, :lens[b]], kn[b, :lens[b]], np.abs(vn[b, :lens[b]]), labels, S, W, rows=r)
             results[("prefill", b)] = assert_matches(f64(out[b, r]), want, f"prefill b={b}", mag, abs_bounds)
+            if raw_name:
+                assert_raw(f64(out[b, r]), want, raw_name + "_prefill")
     check_cache_image(cache, k, v, lens, labels, S, W)
 
     kall = [kn[b, :lens[b]] for b in range(B)]
@@ -126,6 +166,8 @@ def run_case(B, Hq, Hkv, d, T, S, W, labels, seq_lens=None, decode_steps=0, sink
             want = oatt.decode_step(dqn[b], kall[b], vall[b], labels, S, W)
             mag = oatt.decode_step(dqn[b], kall[b], np.abs(vall[b]), labels, S, W)
             results[("decode", step, b)] = assert_matches(f64(dout[b]), want, f"decode step={step} b={b}", mag, abs_bounds)
+            if raw_name:
+                assert_raw(f64(dout[b]), want, raw_name + "_decode")
     cache.check()
     if decode_steps:
         new_lens = [L + decode_steps for L in lens]

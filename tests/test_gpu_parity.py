@@ -16,7 +16,7 @@ def test_tiny_workload_prefill_then_32_decode_steps():
     KV head 0 retrieval, KV head 1 streaming with S=16, W=128; sink key x8."""
     wl = TINY
     run_case(wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.d_head, wl.prefill_len, wl.sink, wl.window,
-             labels_for(wl), decode_steps=wl.decode_steps, sink_scale=wl.sink_scale)
+             labels_for(wl), decode_steps=wl.decode_steps, sink_scale=wl.sink_scale, raw_name="tiny")
 
 
 CASES = {
