@@ -5,7 +5,10 @@ One "step" is one decode step of the Llama-3-8B-shaped decode workload
 tokens, 4 of 8 KV heads streaming with S=128, W=4096): the headline is
 decode attention us/step and its HBM GB/s. The same run times the
 Qwen2.5-7B-shaped 32K prefill (28 / 4 heads, 2 streaming, S=128, W=2048) for
-prefill attention TFLOP/s, reported in the "prefill" object.
+prefill attention TFLOP/s, reported in the "prefill" object, and, with
+short timed regions, the two other workloads: two layers of the 28-layer
+Qwen2.5-7B-shaped stack at 256K (per-layer prefill and decode, KV bytes;
+"stack_256k") and the 12-point ragged decode sweep ("ragged_sweep").
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
 
@@ -30,6 +33,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "decode attn µs/step & HBM GB/s @128K ctx; prefill attn TFLOP/s @32K"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e, nominal (context beside the measured copy rate)
 
 
 def load_peaks():
@@ -362,7 +366,6 @@ def run_native(args):
         pcache.prefill(q, k, v, pout)
         pev[s + 1].record(stream)
     barrier()
-    clock_info = clocks.stop() if clocks else None
     pre_ms = max_over_ranks(pev[0].elapsed_time(pev[Kp])) / Kp
     pcache.check()
     flops = prefill_flops(pwl, plabels, T)
@@ -417,6 +420,21 @@ def run_native(args):
     evict_flops = prefill_flops(pwl, plabels, T, chunk=C)
     del chunks, couts
 
+    # ---------------- the other two workloads: the 256K stack (two layers) and
+    # the ragged decode sweep, with short timed regions
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    tf_peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    stack = ragged = None
+    if not args.no_extra_workloads:
+        del q, k, v
+        torch.cuda.empty_cache()
+        barrier()
+        stack = stack_leg(aoh, torch, args.extra_steps, W, args.stack_layers, 2, tf_peak, hbm_peak)
+        barrier()
+        ragged = ragged_leg(aoh, torch, args.extra_steps, W, hbm_peak)
+        barrier()
+    clock_info = clocks.stop() if clocks else None
+
     # ---------------- cpu baseline (oracle on a bounded sample), rank 0 only
     cpu = pcpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -425,8 +443,6 @@ def run_native(args):
 
     if rank != 0:
         return
-    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
-    tf_peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
     line = {
         "metric": METRIC,
         "value": round(dec_us_step, 3),
@@ -453,7 +469,11 @@ def run_native(args):
                    "bytes_per_step": int(avg_bytes), "kernel_us_median": round(statistics.median(per_step_ms) * 1000, 3)},
         "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                      "frac": round(dec_gbs / hbm_peak, 4), "traffic": traffic_for(decode_kernel_key(wl)),
-                     "peak_note": f"{peak_note} HBM copy bandwidth; kernel: " + decode_kernel_name(wl)},
+                     "peak_note": f"peak = {peak_note} HBM copy bandwidth (a read+write copy; decode only reads, "
+                                  f"so frac is a ratio to the measured copy rate and may pass 1); kernel: "
+                                  + decode_kernel_name(wl),
+                     "nominal_peak": NOMINAL_HBM_GBS,
+                     "frac_of_nominal": round(dec_gbs / NOMINAL_HBM_GBS, 4)},
         "prefill": {"ms": round(pre_ms, 3), "tflops": round(pre_tflops, 2), "flops": flops, "steps": Kp,
                     "tflops_all_ranks": round(pre_tflops_total, 2),
                     "roofline": {"bound": "tensor", "achieved": round(pre_tflops, 2), "peak": tf_peak,
@@ -471,6 +491,8 @@ def run_native(args):
                                            "the W tokens before their chunk and the chunk (attended pairs counted "
                                            "under that rule)"},
         "h2share": h2,
+        "stack_256k": stack,
+        "ragged_sweep": ragged,
         "e2e": {"value": round(e2e_us, 3), "unit": "us/step", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": K,
         "clocks": clock_info,
@@ -702,20 +724,13 @@ def _decode_timing(aoh, torch, cache, wl, steps, warmup):
     return e0.elapsed_time(e1) * 1000.0 / steps, before
 
 
-def run_ragged(args):
-    """Decode of 64 sequences with lengths uniform in [4K, 32K], S = 64:
-    streaming fraction x window sweep (one JSON line, one entry per point)."""
+def ragged_leg(aoh, torch, steps, warmup, hbm):
+    """Decode of 64 sequences with lengths uniform in [4K, 32K], S = 64, over
+    the sweep of streaming fraction x window: one entry per point, with the
+    HBM fraction of its algorithmic bytes."""
     import dataclasses
 
-    import torch
-
-    from paper_2608_06849_gb300 import aoh
-    from paper_2608_06849_gb300 import build as aoh_build
     from paper_2608_06849_gb300.workloads import RAGGED, labels_for, randn_bf16, seq_lens
-    aoh_build.build()
-    aoh.load()
-    peaks, note = load_peaks()
-    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     lens = seq_lens(RAGGED)
     T = max(lens)
     B, Hkv, D = RAGGED.batch, RAGGED.n_kv_heads, RAGGED.d_head
@@ -726,82 +741,127 @@ def run_ragged(args):
         for W in (512, 2048, 8192):
             wl = dataclasses.replace(RAGGED, n_streaming=int(frac * Hkv), window=W)
             labels = labels_for(wl)
-            cache = aoh.Cache(B, wl.n_q_heads, Hkv, D, T + args.steps + args.warmup + 4, wl.sink, W, labels)
+            cache = aoh.Cache(B, wl.n_q_heads, Hkv, D, T + steps + warmup + 4, wl.sink, W, labels)
             cache.prefill(None, kfill, vfill, None, seq_lens=lens)
-            us, before = _decode_timing(aoh, torch, cache, wl, args.steps, args.warmup)
+            us, before = _decode_timing(aoh, torch, cache, wl, steps, warmup)
             nbytes = decode_bytes(before, labels, wl)
             points.append({"streaming_frac": frac, "window": W, "us_per_step": round(us, 2),
                            "bytes_per_step": nbytes, "hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
                            "frac_of_peak": round(nbytes / (us * 1e-6) / 1e9 / hbm, 4)})
             cache.close()
-    print(json.dumps({"workload": f"{RAGGED.name}: B={B} Hq={RAGGED.n_q_heads} Hkv={Hkv} d={D} "
-                                  f"lens uniform [4096, 32768] seed {RAGGED.seed} S={RAGGED.sink}",
-                      "metric": "decode attn us/step and HBM GB/s", "steps": args.steps, "warmup": args.warmup,
-                      "peak_hbm_gbs": hbm, "peak_note": note, "sweep": points,
-                      "cpu_baseline": None if args.no_cpu_baseline else dict(
-                          oracle_decode_layer(dataclasses.replace(RAGGED, n_streaming=Hkv // 2, window=2048),
-                                              labels_for(dataclasses.replace(RAGGED, n_streaming=Hkv // 2)),
-                                              list(lens), budget_s=5.0),
-                          point="streaming_frac 0.5, window 2048")}))
+    del kfill, vfill
+    torch.cuda.empty_cache()
+    return {"workload": f"{RAGGED.name}: B={B} Hq={RAGGED.n_q_heads} Hkv={Hkv} d={D} "
+                        f"lens uniform [4096, 32768] seed {RAGGED.seed} S={RAGGED.sink}",
+            "steps": steps, "warmup": warmup, "peak_hbm_gbs": hbm, "sweep": points,
+            "frac_range": [min(p["frac_of_peak"] for p in points), max(p["frac_of_peak"] for p in points)]}
 
 
-def run_stack(args):
-    """One layer of the 28-layer Qwen2.5-7B-shaped stack at 256K: per-layer
-    prefill latency and decode latency, and the whole stack's KV bytes
-    against the all-retrieval layout."""
+def run_ragged(args):
+    """The ragged sweep alone (one JSON line), with the oracle's time on one
+    sweep point."""
+    import dataclasses
+
     import torch
 
     from paper_2608_06849_gb300 import aoh
     from paper_2608_06849_gb300 import build as aoh_build
-    from paper_2608_06849_gb300.workloads import STACK_256K, labels_for, prefill_inputs
+    from paper_2608_06849_gb300.workloads import RAGGED, labels_for, seq_lens
     aoh_build.build()
     aoh.load()
     peaks, note = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    res = ragged_leg(aoh, torch, args.steps, args.warmup, hbm)
+    res.update({"metric": "decode attn us/step and HBM GB/s", "peak_note": note})
+    half = dataclasses.replace(RAGGED, n_streaming=RAGGED.n_kv_heads // 2, window=2048)
+    res["cpu_baseline"] = None if args.no_cpu_baseline else dict(
+        oracle_decode_layer(half, labels_for(half), seq_lens(RAGGED), budget_s=5.0),
+        point="streaming_frac 0.5, window 2048")
+    print(json.dumps(res))
+
+
+def stack_leg(aoh, torch, steps, warmup, layers, prefill_reps, tf_peak, hbm, cpu=False):
+    """Layers of the 28-layer Qwen2.5-7B-shaped stack at 256K (each layer its
+    own labels and inputs): per layer, the 256K prefill and `steps` decode
+    steps after it; the whole stack's KV bytes against the all-retrieval
+    layout. Per-layer figures with their roofline fractions."""
+    from paper_2608_06849_gb300.workloads import STACK_256K, labels_for, prefill_inputs
     wl = STACK_256K
     T = wl.prefill_len
-    labels = labels_for(wl, layer=0)
-    q, k, v = prefill_inputs(wl, device="cuda")
-    cache = aoh.Cache(1, wl.n_q_heads, wl.n_kv_heads, wl.d_head, T + args.steps + args.warmup + 4, wl.sink,
-                      wl.window, labels)
-    out = torch.empty_like(q)
-    for _ in range(2):
+    per_layer = []
+    cpu_base = None
+    for layer in range(layers):
+        labels = labels_for(wl, layer=layer)
+        q, k, v = prefill_inputs(wl, device="cuda", seed_offset=layer)
+        cache = aoh.Cache(1, wl.n_q_heads, wl.n_kv_heads, wl.d_head, T + steps + warmup + 4, wl.sink, wl.window,
+                          labels)
+        out = torch.empty_like(q)
         cache.reset()
         cache.prefill(q, k, v, out)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    reps = 3
-    torch.cuda.synchronize()
-    e0.record()
-    for _ in range(reps):
-        cache.reset()
-        cache.prefill(q, k, v, out)
-    e1.record()
-    torch.cuda.synchronize()
-    cache.check()
-    pre_ms = e0.elapsed_time(e1) / reps
-    flops = prefill_flops(wl, labels, T)
-    del q, out
-    us, before = _decode_timing(aoh, torch, cache, wl, args.steps, args.warmup)
-    nbytes = decode_bytes(before, labels, wl)
-    cfg = cache.cfg
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(prefill_reps):
+            cache.reset()
+            cache.prefill(q, k, v, out)
+        e1.record()
+        torch.cuda.synchronize()
+        cache.check()
+        pre_ms = e0.elapsed_time(e1) / prefill_reps
+        flops = prefill_flops(wl, labels, T)
+        del q, out, k, v
+        us, before = _decode_timing(aoh, torch, cache, wl, steps, warmup)
+        nbytes = decode_bytes(before, labels, wl)
+        cache.close()
+        torch.cuda.empty_cache()
+        per_layer.append({"layer": layer, "labels": labels, "prefill_ms": round(pre_ms, 3),
+                          "prefill_tflops": round(flops / (pre_ms * 1e-3) / 1e12, 1),
+                          "prefill_frac_of_peak": round(flops / (pre_ms * 1e-3) / 1e12 / tf_peak, 4),
+                          "decode_us_per_step": round(us, 2), "decode_bytes_per_step": nbytes,
+                          "decode_hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
+                          "decode_frac_of_peak": round(nbytes / (us * 1e-6) / 1e9 / hbm, 4)})
+        if cpu and layer == 0:
+            cpu_base = {"decode": oracle_decode_layer(wl, labels, before, budget_s=5.0),
+                        "prefill": oracle_prefill_sample(8.0, wl, labels)}
+    cfg = aoh.make_config(1, wl.n_q_heads, wl.n_kv_heads, wl.d_head, T + wl.decode_steps, wl.sink, wl.window)
     kv_aoh = sum(aoh.aoh_cache_bytes(cfg, labels_for(wl, layer=L)) for L in range(wl.layers))
     kv_full = wl.layers * aoh.aoh_cache_bytes(cfg, [0] * wl.n_kv_heads)
-    cache.close()
+    n = len(per_layer)
+    pre_ms = sum(x["prefill_ms"] for x in per_layer) / n
+    dec_us = sum(x["decode_us_per_step"] for x in per_layer) / n
+    res = {
+        "workload": f"{wl.name}: {wl.layers} layers x (Hq={wl.n_q_heads} Hkv={wl.n_kv_heads} d={wl.d_head}), "
+                    f"T={T} (+{wl.decode_steps} decode), 2 of 4 KV heads streaming per layer, S={wl.sink} "
+                    f"W={wl.window}; {n} layers timed",
+        "layers_timed": per_layer, "prefill_reps": prefill_reps, "decode_steps": steps, "decode_warmup": warmup,
+        "prefill_ms_per_layer": round(pre_ms, 3),
+        "prefill_frac_of_peak": round(sum(x["prefill_frac_of_peak"] for x in per_layer) / n, 4),
+        "decode_us_per_layer_step": round(dec_us, 2),
+        "decode_frac_of_peak": round(sum(x["decode_frac_of_peak"] for x in per_layer) / n, 4),
+        "stack_estimate": {"prefill_s": round(wl.layers * pre_ms / 1000, 3),
+                           "decode_ms_per_token": round(wl.layers * dec_us / 1000, 3)},
+        "kv_bytes_stack": kv_aoh, "kv_bytes_all_retrieval": kv_full, "kv_ratio": round(kv_full / kv_aoh, 4),
+        "peaks": {"bf16_tflops": tf_peak, "hbm_gbs": hbm}}
+    if cpu_base is not None:
+        res["cpu_baseline"] = cpu_base
+    return res
+
+
+def run_stack(args):
+    """The 256K stack alone (one JSON line), with the oracle's time on layer 0."""
+    import torch
+
+    from paper_2608_06849_gb300 import aoh
+    from paper_2608_06849_gb300 import build as aoh_build
+    aoh_build.build()
+    aoh.load()
+    peaks, note = load_peaks()
     tf_peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
-    print(json.dumps({
-        "workload": f"{wl.name}: {wl.layers} layers x (Hq={wl.n_q_heads} Hkv={wl.n_kv_heads} d={wl.d_head}), "
-                    f"T={T}, 2 of 4 KV heads streaming per layer, S={wl.sink} W={wl.window}; one layer timed",
-        "prefill_ms_per_layer": round(pre_ms, 3), "prefill_tflops": round(flops / (pre_ms * 1e-3) / 1e12, 1),
-        "prefill_frac_of_peak": round(flops / (pre_ms * 1e-3) / 1e12 / tf_peak, 4),
-        "decode_us_per_layer_step": round(us, 2), "decode_hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
-        "decode_frac_of_peak": round(nbytes / (us * 1e-6) / 1e9 / hbm, 4),
-        "stack_estimate": {"prefill_s": round(wl.layers * pre_ms / 1000, 3),
-                           "decode_ms_per_token": round(wl.layers * us / 1000, 3)},
-        "kv_bytes_stack": kv_aoh, "kv_bytes_all_retrieval": kv_full, "kv_ratio": round(kv_full / kv_aoh, 4),
-        "peak_note": note,
-        "cpu_baseline": None if args.no_cpu_baseline else {
-            "decode": oracle_decode_layer(wl, labels, before, budget_s=5.0),
-            "prefill": oracle_prefill_sample(8.0, wl, labels)}}))
+    res = stack_leg(aoh, torch, args.steps, args.warmup, args.stack_layers, 3, tf_peak, hbm,
+                    cpu=not args.no_cpu_baseline)
+    res["peak_note"] = note
+    print(json.dumps(res))
 
 
 def run_graph(args):
@@ -1023,6 +1083,11 @@ def main():
     ap.add_argument("--decode-batch", type=int, default=None, help="smaller decode batch (profiling runs)")
     ap.add_argument("--decode-ctx", type=int, default=None, help="smaller decode context (profiling runs)")
     ap.add_argument("--prefill-len", type=int, default=None, help="shorter prefill (profiling runs)")
+    ap.add_argument("--stack-layers", type=int, default=2, help="layers of the 256K stack timed")
+    ap.add_argument("--extra-steps", type=int, default=16,
+                    help="timed decode steps of the stack and ragged legs in the default run")
+    ap.add_argument("--no-extra-workloads", action="store_true",
+                    help="default run without the 256K stack and ragged sweep legs (profiling runs)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "native":
         args.warmup = 3
