@@ -200,11 +200,8 @@ aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* 
  * Retrieval head i of sequence b attends to the first min(top_k, t + 1)
  * entries of its list; entries outside [0, t] are clamped into it (the
  * reads stay in bounds, the result is then unspecified). d_head 128 runs on
- * the tensor cores with the borrowed rows gathered by TMA; d_head 64 on the
- * CUDA-core kernel. The TMA gathers address rows with 32-bit coordinates:
- * when B * n_r * 2 * max_seq >= 2^31 a d_head 128 cache also takes the
- * CUDA-core kernel, which supports groups of 1, 2, 4, 7 and 8 (other groups
- * return UNSUPPORTED).
+ * the tensor cores, the borrowed rows copied by four gather warps; d_head 64
+ * on the CUDA-core kernel.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,

@@ -105,8 +105,6 @@ void aoh::record_error(const char* msg) { g_last_error = msg; }
 
 struct aoh_cache {
   CUtensorMap tcr, tcs;  // cache regions for TMA (built once: the buffer does not move)
-  CUtensorMap tcg;       // retrieval rows for row gathers (valid when has_tcg)
-  bool has_tcg = false;
   aoh_config cfg;
   CacheGeom geom;
   std::vector<uint8_t> labels;
@@ -250,7 +248,6 @@ aoh_status aoh_cache_init(const aoh_config* cfg, const uint8_t* head_labels, voi
   h->d_done = h->d_gcounters + n_gcnt;
   h->d_err = h->d_done + 32;
   h->d_partials = reinterpret_cast<float*>(base + 2 * n_lens + n_cnt + n_gcnt + 64);
-  h->has_tcg = make_gather_map(&h->tcg, h->geom, h->kv);
   if (!make_cache_region_maps(&h->tcr, &h->tcs, h->geom, h->kv)) {
     cudaFree(h->meta);
     delete h;
@@ -449,7 +446,6 @@ aoh_status prepare_decode(const void* q, const void* k_new, const void* v_new, a
   }
   a.tcr = cache->tcr;
   a.tcs = cache->tcs;
-  if (cache->has_tcg) a.tcg = cache->tcg;
   a.geom = g;
   a.q = q;
   a.k_new = k_new;
@@ -520,9 +516,9 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
   const aoh_status st = prepare_decode(q, k_new, v_new, cache, out, a, total);
   if (st != AOH_OK) return st;
   const CacheGeom& g = cache->geom;
-  // d_head 128: the tcgen05 kernel gathers the borrowed rows (tile::gather4),
-  // a gathered row weighing kGatherWeight contiguous rows in the CTA split
-  const bool tc = decode_uses_tc(g.D, g.G) && (g.n_r == 0 || cache->has_tcg);
+  // d_head 128: the tcgen05 kernel's gather warps copy the borrowed rows, a
+  // gathered row weighing kGatherWeight contiguous rows in the CTA split
+  const bool tc = decode_uses_tc(g.D, g.G);
   if (!tc && !decode_cc_supported(g.D, g.G))
     return fail(AOH_ERR_UNSUPPORTED, "group size not compiled for the reuse step");
   if (top_k < 1) return fail(AOH_ERR_INVALID, "top_k must be >= 1");

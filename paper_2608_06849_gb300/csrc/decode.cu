@@ -3,8 +3,7 @@
 // attend over their whole history, streaming KV heads over their S sink + W
 // window slots. This kernel serves d_head 64 (d_head 128 runs on the tensor
 // cores, decode_tc.cu), including the d_head 64 H2Share reuse step, whose
-// retrieval rows are borrowed positions gathered one row at a time (and d_head
-// 128 when the tcgen05 kernel's gather map cannot address the cache).
+// retrieval rows are borrowed positions gathered one row at a time.
 //
 // One CTA = one (sequence b, KV head, split) work unit; a split is a
 // contiguous range of cache rows. All G query heads of the GQA group are

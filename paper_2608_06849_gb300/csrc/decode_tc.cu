@@ -14,7 +14,7 @@
 // CTAs, the partial format and the merge are those of the CUDA-core kernel
 // (decode_common.cuh); one CTA per SM.
 //
-// Warp roles (192 threads):
+// Warp roles (192 threads; 320 in the reuse step's variant):
 //   warps 0-3  softmax: thread t owns key t of the tile (TMEM lane t). It
 //              reads its 16 scores, hides keys past the tile's valid rows,
 //              takes the per-head tile maximum (warp redux, then the four
@@ -27,13 +27,13 @@
 //              zero weight times a NaN is NaN.
 //   warp 4     TMA producer: K and V tiles of one (sequence, KV head) region
 //              into a 3-stage ring (4D tensor maps over the cache regions,
-//              128-byte swizzle, rows past the region read as zeros). In the
-//              H2Share reuse step a retrieval item's rows are borrowed
-//              positions: the warp's lanes gather them four at a time
-//              (tile::gather4 over a one-row-box map of all retrieval rows),
-//              and the CTAs split the step's rows with each gathered row
-//              weighing kGatherWeight contiguous rows (a row gather costs
-//              more than its share of a streamed tile).
+//              128-byte swizzle, rows past the region read as zeros).
+//   warps 6-9  (the H2Share reuse step's variant) gather warps: a retrieval
+//              item's rows are borrowed positions, which these warps copy
+//              with 16-byte cp.async copies into the same swizzled ring, 32
+//              rows of each tile per warp; the CTAs split the step's rows
+//              with each gathered row weighing kGatherWeight contiguous rows
+//              (a row gather costs more than its share of a streamed tile).
 //   warp 5     TMEM owner and MMA issuer. Loads each item's Q into one of two
 //              swizzled buffers, writes the new token's K/V row over its
 //              (stale) cache row in the landed tile and appends it to the
@@ -53,7 +53,8 @@ constexpr int kD = 128;
 constexpr int kBN = 128;                   // keys per tile
 constexpr int kN = 16;                     // N of both MMAs (query heads, padded)
 constexpr int kNS = 3;                     // ring stages
-constexpr int kThreads = 192;
+constexpr int kThreads = 192;              // warps 0-5 (see the file comment)
+constexpr int kGatherWarps = 4;            // warps 6-9 of the H2Share reuse variant
 constexpr int kSoftmaxThreads = 128;
 constexpr uint32_t kTmemCols = 64;         // S[0] [0,16), S[1] [16,32), O [32,48)
 constexpr uint32_t kOcol = 32;
@@ -69,21 +70,25 @@ constexpr int OFF_RED = OFF_P + 2 * kOpBuf;   // [2][4][16] warp maxima, [4][16]
 constexpr int OFF_MS = OFF_RED + (2 * 64 + 64) * 4;
 constexpr int MS_FLOATS = 1024;               // merge scratch
 constexpr int OFF_BAR = OFF_MS + MS_FLOATS * 4;
-constexpr int NBAR = 2 * kNS + 2 + 2 + 2 + 2 + 1 + 1;
+constexpr int NBAR = 3 * kNS + 2 + 2 + 2 + 2 + 1 + 1;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
 constexpr int kLensCap = 2048;                // sequence lengths mirrored in shared memory
 constexpr int OFF_LENS = OFF_MISC + 64;
-constexpr int OFF_PATCH = OFF_LENS + kLensCap * 4;  // [kNS][4] new-token slot masks (gathered tiles)
-constexpr int SMEM = OFF_PATCH + kNS * 16 + 1024;
+constexpr int SMEM = OFF_LENS + kLensCap * 4 + 1024;
 constexpr uint32_t IDESC_S = idesc_bf16(kBN, kN, false, false);
 constexpr uint32_t IDESC_PV = idesc_bf16(kD, kN, false, true);
 static_assert(SMEM <= 232448, "shared memory");
 static_assert(OFF_Q % 1024 == 0 && OFF_P % 1024 == 0, "operand alignment");
-static_assert(kThreads * 8 <= kNS * kStage, "scan scratch");
+static_assert((kThreads + 32 * kGatherWarps) * 8 <= kNS * kStage, "scan scratch");
 
-template <int G>
-__global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
+// GATHER: the H2Share reuse variant, whose four gather warps copy the borrowed
+// rows of retrieval items (a.idx != nullptr); the producer warp then loads
+// only the contiguous (streaming) tiles.
+template <int G, bool GATHER>
+__global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1)
+    decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
   static_assert(G >= 1 && G <= kN, "group size");
+  constexpr int NT = kThreads + (GATHER ? 32 * kGatherWarps : 0);
   static_assert(2 * (dec::kGroup + 8) * G + 2 * G <= MS_FLOATS, "merge scratch");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
@@ -93,9 +98,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   float* red = reinterpret_cast<float*>(smem + OFF_RED);  // [2][4][16]
   float* lsum = red + 2 * 64;                             // [4][16]
   float* ms = reinterpret_cast<float*>(smem + OFF_MS);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + OFF_BAR);  // [kNS] a TMA-loaded tile landed
   uint64_t* empty = full + kNS;
-  uint64_t* s_full = empty + kNS;   // [2] S(j) in TMEM
+  uint64_t* gfull = empty + kNS;    // [kNS] a gathered tile landed (reuse variant)
+  uint64_t* s_full = gfull + kNS;   // [2] S(j) in TMEM
   uint64_t* s_free = s_full + 2;    // [2] S(j) read by the softmax
   uint64_t* p_full = s_free + 2;    // [2] P(j) written
   uint64_t* p_free = p_full + 2;    // [2] O += P(j) V(j) done
@@ -106,7 +112,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   long long* sh64 = reinterpret_cast<long long*>(smem + OFF_MISC + 8);  // [0] total, [1] first offset
   int* sh32 = reinterpret_cast<int*>(sh64 + 2);                         // [0] first item, [1] merge flag
   int* lens_s = reinterpret_cast<int*>(smem + OFF_LENS);
-  uint32_t* patch = reinterpret_cast<uint32_t*>(smem + OFF_PATCH);
 
   const CacheGeom& g = a.geom;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -117,13 +122,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   // Prologue that touches no global memory; it may overlap the tail of the
   // previous kernel on the stream (programmatic dependent launch).
   // Q and P rows >= G stay zero for the whole launch
-  for (int i = threadIdx.x; i < 4 * kOpBuf / 16; i += kThreads)
+  for (int i = threadIdx.x; i < 4 * kOpBuf / 16; i += NT)
     reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0, 0, 0, 0);
   fence_proxy_async_smem();
   if (threadIdx.x == 0) {
     for (int s = 0; s < kNS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
+      mbar_init(&gfull[s], kGatherWarps);
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&s_full[x], 1);
@@ -152,10 +158,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   // advances them), so every role reads this copy
   const int* ls = g.B <= kLensCap ? lens_s : nullptr;
   if (ls != nullptr) {
-    for (int i = threadIdx.x; i < g.B; i += kThreads) lens_s[i] = __ldcg(&a.lens[i]);
+    for (int i = threadIdx.x; i < g.B; i += NT) lens_s[i] = __ldcg(&a.lens[i]);
     __syncthreads();
   }
-  dec::find_cta_range<kThreads>(a, reinterpret_cast<long long*>(sKV), sh64, sh32, ls);
+  dec::find_cta_range<NT>(a, reinterpret_cast<long long*>(sKV), sh64, sh32, ls);
   __syncthreads();
   const long long total = sh64[0];
   const long long start = (long long)p * total / P;
@@ -165,20 +171,76 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
 
   if (warp == 4) {
     // ------------------------------------------------------------ producer
-    // Contiguous items: lane 0 loads 128-row K and V tiles of the region.
-    // Retrieval items of the H2Share reuse step (a.idx): every lane gathers
-    // four of a tile's 128 borrowed rows (tile::gather4 over the gather map,
-    // one instruction per row quad, 64-column half and K or V), with the
-    // tile's indices loaded two tiles ahead. Slots past the item's rows read
-    // row 0 (the softmax gives them zero weight); slots holding the new
-    // token (position t, not in the cache yet) read row 0 too and are
-    // listed in the stage's patch mask for the MMA warp to overwrite.
-    if (lane == 0) {
-      if (g.n_r > 0) prefetch_tmap(a.idx ? &a.tcg : &a.tcr);
+    // Lane 0 loads 128-row K and V tiles of the region (4D tensor maps over
+    // the cache regions, 128-byte swizzle). In the reuse variant the gather
+    // warps issue every tile instead (see below) and this warp idles.
+    if (!GATHER && lane == 0) {
+      if (g.n_r > 0) prefetch_tmap(&a.tcr);
       if (g.n_s > 0) prefetch_tmap(&a.tcs);
+      int it = 0;
+      bool ok = true;
+      long long off = first_off;
+      for (int id = first_id; id < n_items && off < end && ok; ++id) {
+        const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
+        const int lo = sp.lo, hi = sp.hi;
+        off += sp.units;
+        if (lo >= hi) continue;
+        const int b = id / HK, k = id - b * HK;
+        const bool strm = k >= g.n_r;
+        const int region = strm ? b * g.n_s + (k - g.n_r) : b * g.n_r + k;
+        const CUtensorMap* map = strm ? &a.tcs : &a.tcr;
+        for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
+          const int st = it % kNS;
+          if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[st], kStage);
+          uint8_t* dst = sKV + st * kStage;
+#pragma unroll
+          for (int sel = 0; sel < 2; ++sel)
+#pragma unroll
+            for (int db = 0; db < 2; ++db)
+              tma_load_4d(dst + sel * kTile + db * kBox, map, db * 64, row0, sel, region, &full[st]);
+        }
+      }
+      // every issued copy lands before the CTA can exit
+      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) wait_bar(&full[j % kNS], (j / kNS) & 1, a.err, abort_flag);
     }
+    __syncwarp();
+  } else if (GATHER && warp >= 6) {
+    // ------------------------------------------------------------ gatherers
+    // The reuse variant's four gather warps issue every tile of the CTA's
+    // range, each of them waiting for every tile's stage to be free, in
+    // order (an mbarrier parity wait is only sound within one phase of the
+    // barrier, so no waiter may skip tiles). Contiguous (streaming) tiles:
+    // lane 0 of warp 6 loads them with the TMA onto full[st]. Retrieval
+    // items: gather warp w copies rows 32 w .. 32 w + 31 of each 128-row tile
+    // of borrowed positions, one row per instruction (lanes 0-15 the 16
+    // chunks of its K row, lanes 16-31 those of its V row) with 16-byte
+    // cp.async copies into the swizzled layout the MMAs read, and the copies
+    // complete on gfull[st]; the new token's row (position t, not in the
+    // cache yet) comes from the step's input. Lane j holds the index of row
+    // 32 w + j, loaded two tiles ahead into one of two registers that
+    // alternate between tiles (a register copy of an in-flight load would
+    // wait for it). Row gathers through the TMA (tile::gather4 or bulk row
+    // copies) ran at about 15 GB/s per SM; cp.async copies scale with the
+    // issuing warps.
+    const int gw = warp - 6;
+    const int half = lane >> 4, ch = lane & 15;
+    const uint32_t dst_lane = half * kTile + (ch >> 3) * kBox;
+    const uint32_t swz = ch & 7;
+    const bool loader = gw == 0 && lane == 0;  // issues the TMA tiles
+    if (loader && g.n_s > 0) prefetch_tmap(&a.tcs);
     int it = 0;
     bool ok = true;
+    uint32_t fpar = 0;  // loader: bit st, parity of stage st's next full[] phase
+    uint32_t mine = 0;  // loader: bit st, stage st's latest tile came through the TMA
+    auto stage_free = [&](int st) -> bool {  // warp-uniform
+      int go = 1;
+      if (lane == 0 && it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) go = 0;
+      return __shfl_sync(0xffffffffu, go, 0) != 0;
+    };
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
       const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
@@ -186,90 +248,83 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       off += sp.units;
       if (lo >= hi) continue;
       const int b = id / HK, k = id - b * HK;
-      const bool strm = k >= g.n_r;
-      const int region = strm ? b * g.n_s + (k - g.n_r) : b * g.n_r + k;
-      if (a.idx != nullptr && !strm) {
-        const int32_t* rowlist = a.idx + ((size_t)b * a.n_idx_groups + a.idx_map[k]) * a.top_k;
-        const int t = dec::seq_len(a, b, ls);
-        const int kbase = region * 2 * g.max_seq, vbase = kbase + g.max_seq;
-        // indices of this tile (nxt) and the next (nx2): each tile's loads
-        // are issued two tiles before its gathers
-        int nxt[4], nx2[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int j0 = lo + 4 * lane + j;
-          nxt[j] = j0 < hi ? __ldg(rowlist + j0) : 0;
-          nx2[j] = j0 + kBN < hi ? __ldg(rowlist + j0 + kBN) : 0;
-        }
-        for (int row0 = lo; row0 < hi; row0 += kBN) {
-          int cr[4];
-          uint32_t newrow[4];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const bool valid = row0 + 4 * lane + j < hi;
-            const int c = min(max(nxt[j], 0), t);
-            newrow[j] = __ballot_sync(0xffffffffu, valid && c == t);
-            cr[j] = valid && c != t ? c : 0;
-            nxt[j] = nx2[j];
-            const int jn = row0 + 2 * kBN + 4 * lane + j;
-            if (jn < hi) nx2[j] = __ldg(rowlist + jn);
-          }
+      if (k >= g.n_r) {
+        const int region = b * g.n_s + (k - g.n_r);
+        for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
           const int st = it % kNS;
-          int go = 1;
-          if (lane == 0) {
-            if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) go = 0;
-            if (go) {
-              // slot 4 * l + j of the tile is bit l of newrow[j]
-#pragma unroll
-              for (int j = 0; j < 4; ++j) patch[st * 4 + j] = newrow[j];
-              mbar_arrive_expect_tx(&full[st], kStage);
-            }
-          }
-          if (!__shfl_sync(0xffffffffu, go, 0)) {
+          if (!stage_free(st)) {
             ok = false;
             break;
           }
-          uint8_t* dst = sKV + st * kStage + 4 * lane * 128;
-#pragma unroll
-          for (int db = 0; db < 2; ++db) {
-            tma_gather4(dst + db * kBox, &a.tcg, db * 64, kbase + cr[0], kbase + cr[1], kbase + cr[2],
-                        kbase + cr[3], &full[st]);
-            tma_gather4(dst + kTile + db * kBox, &a.tcg, db * 64, vbase + cr[0], vbase + cr[1], vbase + cr[2],
-                        vbase + cr[3], &full[st]);
-          }
-          ++it;
-        }
-      } else {
-        if (lane == 0) {
-          const CUtensorMap* map = strm ? &a.tcs : &a.tcr;
-          for (int row0 = lo; row0 < hi; row0 += kBN) {
-            const int st = it % kNS;
-            if (it >= kNS && !wait_bar(&empty[st], ((it / kNS) & 1) ^ 1, a.err, abort_flag)) {
-              ok = false;
-              break;
-            }
+          if (loader) {
             mbar_arrive_expect_tx(&full[st], kStage);
             uint8_t* dst = sKV + st * kStage;
 #pragma unroll
             for (int sel = 0; sel < 2; ++sel)
 #pragma unroll
               for (int db = 0; db < 2; ++db)
-                tma_load_4d(dst + sel * kTile + db * kBox, map, db * 64, row0, sel, region, &full[st]);
-            ++it;
+                tma_load_4d(dst + sel * kTile + db * kBox, &a.tcs, db * 64, row0, sel, region, &full[st]);
+            fpar ^= 1u << st;
+            mine |= 1u << st;
           }
         }
-        // lane 0 alone advanced the ring counter and saw the waits
-        it = __shfl_sync(0xffffffffu, it, 0);
-        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        continue;
+      }
+      const int32_t* rowlist = a.idx + ((size_t)b * a.n_idx_groups + a.idx_map[k]) * a.top_k;
+      const int t = dec::seq_len(a, b, ls);
+      const bf16* src_base =
+          static_cast<const bf16*>(a.kv) + g.r_region(b, k) + (half ? (size_t)g.max_seq * kD : 0) + ch * 8;
+      const bf16* src_new =
+          static_cast<const bf16*>(half ? a.v_new : a.k_new) + ((size_t)b * g.Hkv + g.r_head[k]) * kD + ch * 8;
+      const int j0 = lo + 32 * gw + lane;
+      int ia = j0 < hi ? __ldg(rowlist + j0) : 0;
+      int ib = j0 + kBN < hi ? __ldg(rowlist + j0 + kBN) : 0;
+      auto gather_tile = [&](int row0, int& buf) -> bool {
+        const int my_row = row0 + 32 * gw + lane < hi ? min(max(buf, 0), t) : -1;
+        const int jn = row0 + 2 * kBN + 32 * gw + lane;
+        buf = jn < hi ? __ldg(rowlist + jn) : 0;
+        const int st = it % kNS;
+        if (!stage_free(st)) return false;
+        uint8_t* tile = sKV + st * kStage + dst_lane;
+#pragma unroll 8
+        for (int j = 0; j < 32; ++j) {
+          const int c = __shfl_sync(0xffffffffu, my_row, j);
+          const int r = 32 * gw + j;
+          if (c >= 0)
+            cp_async16(tile + r * 128 + ((swz ^ (uint32_t)(r & 7)) << 4),
+                       c == t ? src_new : src_base + (size_t)c * kD);
+        }
+        cp_async_mbar_arrive(&gfull[st]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&gfull[st]);
+        if (loader) mine &= ~(1u << st);
+        ++it;
+        return true;
+      };
+      for (int row0 = lo; row0 < hi; row0 += 2 * kBN) {
+        if (!gather_tile(row0, ia)) {
+          ok = false;
+          break;
+        }
+        if (row0 + kBN >= hi) break;
+        if (!gather_tile(row0 + kBN, ib)) {
+          ok = false;
+          break;
+        }
       }
     }
-    // every issued copy lands before the CTA can exit
-    if (lane == 0)
-      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) wait_bar(&full[j % kNS], (j / kNS) & 1, a.err, abort_flag);
+    // every copy issued here lands before the CTA can exit: the cp.async
+    // copies, and the latest TMA tile of each stage
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    if (loader)
+      for (int st = 0; st < kNS; ++st)
+        if (mine & (1u << st)) wait_bar(&full[st], ((fpar >> st) & 1) ^ 1, a.err, abort_flag);
+    __syncwarp();
   } else if (warp == 5) {
     // ------------------------------------------------------------ MMA issuer
     const uint32_t kv_addr = smem_u32(sKV), q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
     int it = 0, item_k = 0, ofw = 0;
+    uint32_t fpar = 0, gpar = 0;  // bit st: parity of stage st's next full[] / gfull[] phase
     bool ok = true;
     struct Pend {
       int it, st, item;
@@ -381,11 +436,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
       }
 
       // H2Share reuse step: this retrieval item's rows are gathered
-      const bool gathered = a.idx != nullptr && !strm;
+      const bool gathered = GATHER && a.idx != nullptr && !strm;
       for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
         const int st = it % kNS;
         const int cnt = min(kBN, hi - row0);
-        wait_warp(&full[st], (it / kNS) & 1);
+        // a tile landed on full[st] (TMA) or gfull[st] (gather warps)
+        wait_warp(gathered ? &gfull[st] : &full[st], ((gathered ? gpar : fpar) >> st) & 1);
+        if (gathered)
+          gpar ^= 1u << st;
+        else
+          fpar ^= 1u << st;
         if (!ok) break;
         auto put_new_row = [&](int r) {  // the new token's K / V chunk into tile slot r
           uint8_t* dst = sKV + st * kStage + (lane < 16 ? 0 : kTile) + (ch >> 3) * kBox + r * 128 +
@@ -393,23 +453,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
           *reinterpret_cast<uint4*>(dst) = nv;
         };
         if (gathered) {
-          // slots that borrow position t; the item's owner of row 0 appends it
-          bool any = false;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            uint32_t m = patch[st * 4 + j];
-            any = any || m != 0u;
-            while (m) {
-              const int l = __ffs(m) - 1;
-              m &= m - 1;
-              put_new_row(4 * l + j);
-            }
-          }
+          // the gather warps wrote this tile with cp.async (generic proxy):
+          // order it before the tensor core's reads; the item's owner of row
+          // 0 appends the new token
           if (row0 == 0) *reinterpret_cast<uint4*>((lane < 16 ? Kc : Vc) + (size_t)xr * kD + ch * 8) = nv;
-          if (any) {
-            fence_proxy_async_smem();
-            __syncwarp();
-          }
+          fence_proxy_async_smem();
+          __syncwarp();
         } else if (xr >= row0 && xr < row0 + cnt) {
           put_new_row(xr - row0);
           *reinterpret_cast<uint4*>((lane < 16 ? Kc : Vc) + (size_t)xr * kD + ch * 8) = nv;  // append
@@ -460,6 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
     // ok: the four warps' common verdict, only ever set at a barrier (so every
     // thread leaves the loops together); local_ok: this thread's waits since
     bool ok = true, local_ok = true;
+    uint32_t fpar = 0, gpar = 0;  // bit st: parity of stage st's next full[] / gfull[] phase
     long long off = first_off;
     for (int id = first_id; id < n_items && off < end && ok; ++id) {
       const dec::Span sp = dec::item_span(a, id, ls, off, start, end);
@@ -477,9 +527,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
         m[h] = -INFINITY;
         l[h] = 0.f;
       }
+      const bool gathered = GATHER && a.idx != nullptr && !strm;
       for (int row0 = lo; row0 < hi; row0 += kBN, ++it) {
         const int x = it & 1, st = it % kNS;
         const int cnt = min(kBN, hi - row0);
+        const uint32_t land_par = ((gathered ? gpar : fpar) >> st) & 1;  // the phase that lands this tile
+        if (gathered)
+          gpar ^= 1u << st;
+        else
+          fpar ^= 1u << st;
         local_ok = wait_bar(&s_full[x], (it >> 1) & 1, a.err, abort_flag) && local_ok;
         tc_fence_after();
         uint32_t v[16];
@@ -546,7 +602,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
         }
         if (!valid) {
           // the tile has landed (its S is complete); zero V row t
-          wait_bar(&full[st], (it / kNS) & 1, a.err, abort_flag);
+          wait_bar(gathered ? &gfull[st] : &full[st], land_par, a.err, abort_flag);
           uint8_t* vr = sKV + st * kStage + kTile + t * 128;
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
@@ -633,11 +689,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(const __grid_con
   if (threadIdx.x == 0) dec::finish_launch(a);
 }
 
-template <int G>
+template <int G, bool GATHER>
 cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    cudaError_t e =
+        cudaFuncSetAttribute(decode_tc_kernel<G, GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -645,7 +702,7 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
   // work on the stream itself (griddepcontrol.wait) after its prologue
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.n_ctas);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kThreads + (GATHER ? 32 * kGatherWarps : 0));
   cfg.dynamicSmemBytes = SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -653,28 +710,12 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<G>, a);
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<G, GATHER>, a);
 }
 
 }  // namespace
 
 bool decode_uses_tc(int D, int G) { return D == kD && ((G >= 1 && G <= 8) || G == 16); }
-
-bool make_gather_map(CUtensorMap* tcg, const CacheGeom& g, const void* kv) {
-  if (g.D != kD || g.n_r <= 0) return false;
-  const long long rows = (long long)g.B * g.n_r * 2 * g.max_seq;
-  if (rows >= (1LL << 31)) return false;  // row coordinates are 32-bit
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
-  cuuint32_t box[2] = {64, 1};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(tcg, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-            const_cast<bf16*>(static_cast<const bf16*>(kv) + g.r_region(0, 0)), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
 
 // One CTA per SM; small steps use fewer, at least 512 rows each.
 // At least 512 rows (four tiles) per CTA, so that small steps keep few
@@ -686,19 +727,25 @@ int decode_tc_ctas(long long total_rows, int num_sms) {
   return p < 1 ? 1 : (int)p;
 }
 
-cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s) {
+template <bool GATHER>
+cudaError_t launch_tc(const DecodeArgs& a, cudaStream_t s) {
   switch (a.geom.G) {
-    case 1: return launch_g<1>(a, s);
-    case 2: return launch_g<2>(a, s);
-    case 3: return launch_g<3>(a, s);
-    case 4: return launch_g<4>(a, s);
-    case 5: return launch_g<5>(a, s);
-    case 6: return launch_g<6>(a, s);
-    case 7: return launch_g<7>(a, s);
-    case 8: return launch_g<8>(a, s);
-    case 16: return launch_g<16>(a, s);
+    case 1: return launch_g<1, GATHER>(a, s);
+    case 2: return launch_g<2, GATHER>(a, s);
+    case 3: return launch_g<3, GATHER>(a, s);
+    case 4: return launch_g<4, GATHER>(a, s);
+    case 5: return launch_g<5, GATHER>(a, s);
+    case 6: return launch_g<6, GATHER>(a, s);
+    case 7: return launch_g<7, GATHER>(a, s);
+    case 8: return launch_g<8, GATHER>(a, s);
+    case 16: return launch_g<16, GATHER>(a, s);
   }
   return cudaErrorInvalidValue;
+}
+
+// The reuse step (a.idx set) launches the variant with gather warps.
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s) {
+  return a.idx != nullptr ? launch_tc<true>(a, s) : launch_tc<false>(a, s);
 }
 
 }  // namespace aoh

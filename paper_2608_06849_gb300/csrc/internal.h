@@ -50,8 +50,6 @@ struct CacheGeom {
 
 struct DecodeArgs {
   CUtensorMap tcr, tcs;  // cache regions (see PrefillTcArgs); read by the tcgen05 kernel
-  CUtensorMap tcg;       // retrieval rows as one [B * n_r * 2 * max_seq][D] matrix, one-row
-                         // box (row gathers of the H2Share reuse step on the tcgen05 kernel)
   CacheGeom geom;
   const void* q;      // [B][Hq][D]
   const void* k_new;  // [B][Hkv][D]
@@ -137,9 +135,6 @@ bool prefill_tc_make_cache_maps(PrefillTcArgs* a, const void* kv);
 // [regions][K, V][capacity rows][D] with box [1][1][128][64] and 128-byte
 // swizzle; a kind with no heads leaves its map untouched.
 bool make_cache_region_maps(CUtensorMap* tcr, CUtensorMap* tcs, const CacheGeom& g, const void* kv);
-// The gather map of DecodeArgs::tcg (d_head 128, retrieval heads present,
-// fewer than 2^31 retrieval rows); false if it cannot be built.
-bool make_gather_map(CUtensorMap* tcg, const CacheGeom& g, const void* kv);
 cudaError_t launch_prefill_tc(const PrefillTcArgs& a, int n_items, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t s);
 // The CUDA-core decode kernel for any supported (D, G) (the H2Share reuse
@@ -165,9 +160,11 @@ int decode_ctas(long long total_rows, int num_sms, int D, int G);
 // The tcgen05 decode kernel serves (D, G) (else the CUDA-core kernel does).
 bool decode_uses_tc(int D, int G);
 // Work units of one gathered row in the reuse step's split on the tcgen05
-// kernel (a 256-byte row gather against a contiguous row's share of a tile
-// stream; measured).
-constexpr int kGatherWeight = 5;
+// kernel: a borrowed K and V row copied by the gather warps against a
+// contiguous row's share of a TMA tile stream (measured at 128K context,
+// top_k 2048: weights 2 / 3 / 4 / 5 gave 79.1 / 65.3 / 66.9 / 75.0 us at
+// B=16, 25.1 / 25.9 / 28.6 us at B=4).
+constexpr int kGatherWeight = 3;
 int decode_tc_ctas(long long total_rows, int num_sms);
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
