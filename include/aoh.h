@@ -360,6 +360,23 @@ aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_la
 aoh_status aoh_decode_step_noalloc_status(uint32_t* flags, void* stream);
 
 /*
+ * Self-test of the allocation-free step's recovery from a bounded-wait
+ * timeout (the paper has no counterpart): the same call and arguments as
+ * aoh_decode_step_noalloc, except that in CTA 0 the softmax warps withhold
+ * their first result, so the MMA warp's wait for it runs out (after about
+ * 2 s) and that CTA stops once its copies and MMAs in flight have landed;
+ * the other CTAs finish. The outputs of this call are unspecified, the new
+ * token may be missing from the cache rows that CTA 0 would have appended,
+ * and the lengths advance as usual. The launch still leaves the static scratch clean, and
+ * aoh_decode_step_noalloc_status() then reports AOH_ERR_TIMEOUT once.
+ * Needs d_head 128 (UNSUPPORTED otherwise). Errors: as
+ * aoh_decode_step_noalloc.
+ */
+aoh_status aoh_decode_step_noalloc_selftest(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
+                                            int32_t* lens, int32_t max_len, const void* q, const void* k_new,
+                                            const void* v_new, void* out, void* stream);
+
+/*
  * Effective-rank head classification (Sec. 4, Eq. 2-6 and Algorithm 1;
  * Appendix "GQA Extension"), computed on the GPU in fp64, for n_layers
  * layers at once. For query head h of a layer, M_h = W_K^T W_Q (Eq. 2, the

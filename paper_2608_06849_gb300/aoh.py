@@ -40,6 +40,7 @@ EXPORTS = [
     "aoh_version",
     "aoh_decode_step_noalloc",
     "aoh_decode_step_noalloc_status",
+    "aoh_decode_step_noalloc_selftest",
     "aoh_classify",
     "aoh_decode_step_anchor",
     "aoh_decode_step_reuse",
@@ -96,6 +97,7 @@ def load():
         "aoh_version": (i32, []),
         "aoh_decode_step_noalloc": (i32, [cfgp, u8p, P, i32p, i32, P, P, P, P, P]),
         "aoh_decode_step_noalloc_status": (i32, [ctypes.POINTER(ctypes.c_uint32), P]),
+        "aoh_decode_step_noalloc_selftest": (i32, [cfgp, u8p, P, i32p, i32, P, P, P, P, P]),
         "aoh_classify": (i32, [P, P, i32, i32, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), u8p, P]),
     }
     for name, (res, args) in sig.items():
@@ -186,9 +188,11 @@ def aoh_decode_step_reuse(q, k_new, v_new, cache, out, indices, top_k, group_map
                                         n_anchor, int(top_k), gm, _stream_ptr(stream)))
 
 
-def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream=None):
+def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream=None,
+                            _selftest=False):
     """The allocation-free decode step: ``kv_buffer`` (CUDA uint8) and ``lens``
-    (CUDA int32 [B], advanced by one on the device) belong to the caller."""
+    (CUDA int32 [B], advanced by one on the device) belong to the caller.
+    ``_selftest`` calls aoh_decode_step_noalloc_selftest instead."""
     if len(labels) != cfg.n_kv_heads:
         raise ValueError(f"labels need {cfg.n_kv_heads} entries (one per KV head)")
     n_s = sum(1 for x in labels if int(x) == STREAMING)
@@ -200,7 +204,8 @@ def aoh_decode_step_noalloc(cfg, labels, kv_buffer, lens, max_len, q, k_new, v_n
         _need(t, name, n)
     if not lens.is_cuda or lens.dtype != torch.int32 or not lens.is_contiguous():
         raise ValueError("lens must be a contiguous int32 CUDA tensor")
-    _check(load().aoh_decode_step_noalloc(
+    fn = load().aoh_decode_step_noalloc_selftest if _selftest else load().aoh_decode_step_noalloc
+    _check(fn(
         ctypes.byref(cfg), _labels_arr(labels), _ptr(kv_buffer, "kv_buffer", torch.uint8),
         ctypes.cast(ctypes.c_void_p(lens.data_ptr()), ctypes.POINTER(ctypes.c_int32)), int(max_len),
         _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"), _ptr(out, "out"), _stream_ptr(stream)))

@@ -91,6 +91,13 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint32_
   }
 }
 
+// Before a CTA exits (or frees TMEM) after a timeout, the copies and MMAs it
+// issued must have landed: wait for them even when another role raised the
+// abort flag (still bounded by kWaitLimitNs).
+__device__ __forceinline__ bool drain_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  return mbar_wait(bar, parity, err);
+}
+
 // ------------------------------------------------------------ bulk copies
 // Non-tensor TMA copy global -> shared; completes `bytes` of tx on `bar`.
 // dst, src 16-byte aligned, bytes a multiple of 16.

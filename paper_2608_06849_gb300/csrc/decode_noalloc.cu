@@ -51,9 +51,12 @@ aoh_status set_err(aoh_status st, const char* msg) {
 
 using namespace aoh;
 
-extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
-                                              int32_t* lens, int32_t max_len, const void* q, const void* k_new,
-                                              const void* v_new, void* out, void* stream) {
+namespace {
+
+// The allocation-free step; stall_cta >= 0 runs the self-test.
+aoh_status noalloc_step(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer, int32_t* lens,
+                        int32_t max_len, const void* q, const void* k_new, const void* v_new, void* out,
+                        void* stream, int stall_cta) {
   if (!cfg || !head_labels || !kv_buffer || !lens || !q || !k_new || !v_new || !out)
     return set_err(AOH_ERR_INVALID, "aoh_decode_step_noalloc: NULL argument");
   const aoh_config& c = *cfg;
@@ -63,6 +66,8 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   const int G = c.n_q_heads / c.n_kv_heads;
   if (!decode_supported(c.d_head, G))
     return set_err(AOH_ERR_UNSUPPORTED, "aoh_decode_step_noalloc: group size not compiled");
+  if (stall_cta >= 0 && !decode_uses_tc(c.d_head, G))
+    return set_err(AOH_ERR_UNSUPPORTED, "aoh_decode_step_noalloc_selftest: needs the d_head 128 tensor-core decode");
   const uintptr_t al = reinterpret_cast<uintptr_t>(kv_buffer) | reinterpret_cast<uintptr_t>(q) |
                        reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new) |
                        reinterpret_cast<uintptr_t>(out);
@@ -159,10 +164,26 @@ extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8
   a.n_ctas = n_ctas;
   a.self_clean = 1;
   a.status = header + kStatusWord;
+  a.stall_cta = stall_cta;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));
   e = launch_decode(a, s);
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: kernel launch failed");
   return AOH_OK;
+}
+
+}  // namespace
+
+extern "C" aoh_status aoh_decode_step_noalloc(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer,
+                                              int32_t* lens, int32_t max_len, const void* q, const void* k_new,
+                                              const void* v_new, void* out, void* stream) {
+  return noalloc_step(cfg, head_labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream, -1);
+}
+
+extern "C" aoh_status aoh_decode_step_noalloc_selftest(const aoh_config* cfg, const uint8_t* head_labels,
+                                                       void* kv_buffer, int32_t* lens, int32_t max_len, const void* q,
+                                                       const void* k_new, const void* v_new, void* out,
+                                                       void* stream) {
+  return noalloc_step(cfg, head_labels, kv_buffer, lens, max_len, q, k_new, v_new, out, stream, 0);
 }
 
 extern "C" aoh_status aoh_decode_step_noalloc_status(uint32_t* flags, void* stream) {

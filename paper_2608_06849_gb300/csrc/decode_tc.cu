@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
         }
       }
       // every issued copy lands before the CTA can exit
-      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) wait_bar(&full[j % kNS], (j / kNS) & 1, a.err, abort_flag);
+      for (int j = it > kNS ? it - kNS : 0; j < it; ++j) drain_wait(&full[j % kNS], (j / kNS) & 1, a.err);
     }
     __syncwarp();
   } else if (GATHER && warp >= 6) {
@@ -318,7 +318,7 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
     asm volatile("cp.async.wait_all;" ::: "memory");
     if (loader)
       for (int st = 0; st < kNS; ++st)
-        if (mine & (1u << st)) wait_bar(&full[st], ((fpar >> st) & 1) ^ 1, a.err, abort_flag);
+        if (mine & (1u << st)) drain_wait(&full[st], ((fpar >> st) & 1) ^ 1, a.err);
     __syncwarp();
   } else if (warp == 5) {
     // ------------------------------------------------------------ MMA issuer
@@ -498,7 +498,7 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
     if (has_pend) issue_pv(pend);
     if (lane == 0) {
       tc_commit(drain);
-      wait_bar(drain, 0, a.err, abort_flag);
+      drain_wait(drain, 0, a.err);
     }
     __syncwarp();
   } else {
@@ -619,7 +619,7 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
         fence_proxy_async_smem();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&p_full[x]);
+        if (lane == 0 && !(it == 0 && p == a.stall_cta)) mbar_arrive(&p_full[x]);
       }
       if (!ok) break;
 

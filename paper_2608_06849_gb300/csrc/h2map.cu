@@ -131,7 +131,7 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
       }
       // no copy may still be in flight when the CTA exits
       for (int j = issued > kStages ? issued - kStages : 0; j < issued; ++j)
-        wait_bar(&full[j % kStages], (j / kStages) & 1, a.err, abort_flag);
+        drain_wait(&full[j % kStages], (j / kStages) & 1, a.err);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -147,6 +147,7 @@ __global__ void __launch_bounds__(kGemmThreads, 2) gemm_kernel(const __grid_cons
         tc_commit(&empty[st]);
       }
       tc_commit(done);
+      drain_wait(done, 0, a.err);  // this warp frees TMEM: its MMAs must be done
     }
   } else {
     // epilogue: warp w reads TMEM lanes 32 * (w % 4) .. + 31, rows of the

@@ -71,6 +71,11 @@ struct DecodeArgs {
   // sticky status (or null): the last CTA ORs in the launch's kErrTimeout /
   // kErrCapacity flags; only the host clears it (allocation-free entry point)
   uint32_t* status = nullptr;
+  // self-test (aoh_decode_step_noalloc_selftest; tcgen05 kernel), -1
+  // otherwise: this CTA's softmax warps withhold their first P, so the MMA
+  // warp's bounded wait for it runs out; every copy still lands, and the
+  // launch's other CTAs finish as usual
+  int stall_cta = -1;
   float scale_log2;   // log2(e) / sqrt(D)
   // H2Share anchor step (tcgen05 kernel): when non-null, every retrieval row's
   // scores (log2 units) go to scores[((b * n_r + i) * G + h) * score_stride + row],

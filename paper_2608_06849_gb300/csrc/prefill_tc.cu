@@ -228,9 +228,9 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
     }
     // every issued copy lands before the CTA can exit
     if (lane == 0) {
-      wait_bar(q_full, 0, a.err, abort_flag);
+      drain_wait(q_full, 0, a.err);
       for (int it = issued > kNS ? issued - kNS : 0; it < issued; ++it)
-        wait_bar(&kv_full[it % kNS], (it / kNS) & 1, a.err, abort_flag);
+        drain_wait(&kv_full[it % kNS], (it / kNS) & 1, a.err);
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -297,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(const __grid_co
         }
       }
       tc_commit(drain);
-      wait_bar(drain, 0, a.err, abort_flag);
+      drain_wait(drain, 0, a.err);
     }
   } else {
     // ------------------------------------------------------------ softmax

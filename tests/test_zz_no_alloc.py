@@ -188,3 +188,44 @@ def test_noalloc_skips_a_full_sequence(labels):
     assert allowed[changed].all(), changed[~allowed[changed]][:8].tolist()
     assert torch.equal(kv[cache.nbytes:], before[cache.nbytes:])
     cache.close()
+
+
+def test_noalloc_recovers_from_a_timeout():
+    """A bounded wait that runs out inside an allocation-free step: the call
+    itself cannot report it (it returns before the kernel runs), so the
+    status word must; and the launch must leave the static scratch clean, or
+    the next step's merges would start from stale arrival counts. The
+    self-test entry point stalls one CTA until its wait gives up (about
+    2 s); the cache and lengths are then restored from copies (the stalled
+    CTA may not have appended the new token) and a plain call must match
+    the oracle."""
+    ensure_lib()
+    B, Hq, Hkv, D, T, S, W, labels = 2, 32, 8, 128, 3000, 64, 500, [1, 0, 0, 1, 1, 0, 0, 1]
+    g = Hq // Hkv
+    wl = Workload("timeout", B, Hq, Hkv, D, T, 1, S, W, sum(labels), seed=13)
+    cache = aoh.Cache(B, Hq, Hkv, D, T + 4, S, W, labels)
+    k = randn_bf16((B, T, Hkv, D), 41, "cuda")
+    v = randn_bf16((B, T, Hkv, D), 42, "cuda")
+    cache.prefill(None, k, v, None)
+    torch.cuda.synchronize()
+    saved = cache.buffer.clone()
+    q, kn, vn = decode_inputs(wl, 0, device="cuda")
+    aoh.aoh_decode_step_noalloc_status()                      # clear anything earlier
+    kv = saved.clone()
+    lens = torch.full((B,), T, dtype=torch.int32, device="cuda")
+    junk = torch.empty_like(q)
+    aoh.aoh_decode_step_noalloc(cache.cfg, labels, kv, lens, T, q, kn, vn, junk, _selftest=True)
+    st, flags = aoh.aoh_decode_step_noalloc_status()
+    assert st == 4 and flags & 1, (st, flags)                  # TIMEOUT, reported once
+    assert aoh.aoh_decode_step_noalloc_status() == (aoh.AOH_OK, 0)
+    assert lens.tolist() == [T + 1] * B
+    kv = saved.clone()
+    lens.fill_(T)
+    out = torch.full_like(q, float("nan"))
+    aoh.aoh_decode_step_noalloc(cache.cfg, labels, kv, lens, T, q, kn, vn, out)
+    torch.cuda.synchronize()
+    assert aoh.aoh_decode_step_noalloc_status() == (aoh.AOH_OK, 0)
+    kk = [np.concatenate([f64(k[b]), f64(kn[b])[None]]) for b in range(B)]
+    vv = [np.concatenate([f64(v[b]), f64(vn[b])[None]]) for b in range(B)]
+    _oracle_check(out, q, kk, vv, labels, S, W, g, "after a timeout")
+    cache.close()
