@@ -461,7 +461,7 @@ __global__ void __launch_bounds__(C::THREADS) decode_kernel(const __grid_constan
 
   // ---- the launch's last CTA advances the lengths
   __syncthreads();
-  if (threadIdx.x == 0) dec::finish_launch(a);
+  if (threadIdx.x == 0) dec::finish_launch(a, nullptr);
 }
 
 template <int D, int G>

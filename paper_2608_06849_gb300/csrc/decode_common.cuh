@@ -339,37 +339,45 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
 // The launch's last CTA advances every sequence length by one, except
 // those of full sequences (seq_full), which it flags with kErrCapacity.
 // Called by thread 0 after a __syncthreads that follows all of the CTA's
-// work. A completed merge leaves its counters at zero; after a timeout some
-// may be left behind, and a self-cleaning launch zeroes them and the error
-// word. The launch's flags (timeout, capacity) are also ORed into the
-// sticky status word when there is one; nothing in a launch clears it.
-__device__ __forceinline__ void finish_launch(const DecodeArgs& a) {
-  __threadfence();
+// work; `lens_s` is the kernel's shared-memory copy of the lengths (or
+// null), which cannot have changed during the launch. A completed merge
+// leaves its counters at zero; after a timeout some may be left behind, and
+// a self-cleaning launch zeroes them and the error word. The launch's flags
+// (timeout, capacity) are also ORed into the sticky status word when there
+// is one; nothing in a launch clears it. Only a launch that reads its flags
+// back (self-cleaning, or with a status word) needs the fences that make
+// every CTA's error-word updates visible to the last one; otherwise the
+// last CTA touches nothing another CTA wrote, and the next launch on the
+// stream starts after this grid has completed.
+__device__ __forceinline__ void finish_launch(const DecodeArgs& a, const int* lens_s) {
+  const bool readback = a.self_clean || a.status != nullptr;
+  if (readback) __threadfence();
   const uint32_t prev = atomicAdd(a.done, 1u);
   if (prev == gridDim.x - 1) {
-    __threadfence();
+    if (readback) __threadfence();
     bool full = false;
     for (int i = 0; i < a.geom.B; ++i) {
-      const int t = a.lens[i];
+      const int t = lens_s ? lens_s[i] : a.lens[i];
       if (seq_full(a.geom, t))
         full = true;
       else
         a.lens[i] = t + 1;
     }
-    const uint32_t e = *reinterpret_cast<volatile uint32_t*>(a.err);
-    const uint32_t flags = e | (full ? kErrCapacity : 0u);
-    if (a.status != nullptr && flags != 0u) atomicOr(a.status, flags);
-    if (a.self_clean) {
-      if (e != 0u) {
+    if (readback) {
+      const uint32_t e = *reinterpret_cast<volatile uint32_t*>(a.err);
+      const uint32_t flags = e | (full ? kErrCapacity : 0u);
+      if (a.status != nullptr && flags != 0u) atomicOr(a.status, flags);
+      if (a.self_clean && e != 0u) {
         const int items = a.geom.B * (a.geom.n_r + a.geom.n_s);
         for (int i = 0; i < items; ++i) a.counters[i] = 0u;
         for (int i = 0; i < 2 * (int)gridDim.x; ++i) a.gcounters[i] = 0u;
         *a.err = 0u;
       }
+      if (!a.self_clean && full) atomicOr(a.err, kErrCapacity);
+      __threadfence();
     } else if (full) {
       atomicOr(a.err, kErrCapacity);
     }
-    __threadfence();
     *a.done = 0u;
   }
 }

@@ -686,7 +686,7 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
   __syncthreads();
   tc_fence_after();
   if (warp == 5) tmem_dealloc(tmem, kTmemCols);
-  if (threadIdx.x == 0) dec::finish_launch(a);
+  if (threadIdx.x == 0) dec::finish_launch(a, ls);
 }
 
 template <int G, bool GATHER>
