@@ -517,7 +517,7 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
   if (st != AOH_OK) return st;
   const CacheGeom& g = cache->geom;
   // d_head 128: the tcgen05 kernel's gather warps copy the borrowed rows, a
-  // gathered row weighing kGatherWeight contiguous rows in the CTA split
+  // gathered row weighing gather_w / ring_w contiguous rows in the CTA split
   const bool tc = decode_uses_tc(g.D, g.G);
   if (!tc && !decode_cc_supported(g.D, g.G))
     return fail(AOH_ERR_UNSUPPORTED, "group size not compiled for the reuse step");
@@ -535,12 +535,13 @@ aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v
   a.idx = g.n_r > 0 ? indices : nullptr;
   a.top_k = top_k;
   a.n_idx_groups = n_anchor_groups;
-  a.gather_w = tc ? kGatherWeight : 1;
+  if (tc) reuse_tc_weights(g.G, &a.gather_w, &a.ring_w);
   // every retrieval item now holds min(top_k, t + 1) rows
   total = 0;
   for (int b = 0; b < g.B; ++b) {
     const long long t1 = cache->lens[b] + 1;
-    total += g.n_r * std::min<long long>(t1, top_k) * a.gather_w + g.n_s * std::min<long long>(t1, g.S + g.W);
+    total += (g.n_r * std::min<long long>(t1, top_k) * a.gather_w +
+              g.n_s * std::min<long long>(t1, g.S + g.W) * a.ring_w + a.ring_w - 1) / a.ring_w;
   }
   a.n_ctas = tc ? decode_tc_ctas(total, cache->num_sms) : decode_cc_ctas(total, cache->num_sms);
   cudaError_t e = tc ? launch_decode_tc(a, (cudaStream_t)stream) : launch_decode_cc(a, (cudaStream_t)stream);

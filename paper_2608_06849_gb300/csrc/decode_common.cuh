@@ -48,10 +48,12 @@ __device__ __forceinline__ int item_rows(const DecodeArgs& a, int id, const int*
   return min(t + 1, g.S + g.W);
 }
 
-// Work units of item `id`: its rows, each gathered row of the reuse step
-// weighted by gather_w. The CTAs split the units equally.
+// Work units of item `id`: its rows, weighted in the reuse step by gather_w
+// (gathered rows) and ring_w (contiguous rows). The CTAs split the units
+// equally.
 __device__ __forceinline__ int item_weight(const DecodeArgs& a, int id) {
-  return (a.idx != nullptr && id % (a.geom.n_r + a.geom.n_s) < a.geom.n_r) ? a.gather_w : 1;
+  if (a.idx == nullptr) return 1;
+  return id % (a.geom.n_r + a.geom.n_s) < a.geom.n_r ? a.gather_w : a.ring_w;
 }
 __device__ __forceinline__ long long item_units(const DecodeArgs& a, int id, const int* lens_s = nullptr) {
   return (long long)item_rows(a, id, lens_s) * item_weight(a, id);

@@ -14,7 +14,8 @@
 // CTAs, the partial format and the merge are those of the CUDA-core kernel
 // (decode_common.cuh); one CTA per SM.
 //
-// Warp roles (192 threads; 320 in the reuse step's variant):
+// Warp roles (192 threads; 704 in the reuse step's variant for G <= 4, 448
+// above):
 //   warps 0-3  softmax: thread t owns key t of the tile (TMEM lane t). It
 //              reads its 16 scores, hides keys past the tile's valid rows,
 //              takes the per-head tile maximum (warp redux, then the four
@@ -28,12 +29,15 @@
 //   warp 4     TMA producer: K and V tiles of one (sequence, KV head) region
 //              into a 3-stage ring (4D tensor maps over the cache regions,
 //              128-byte swizzle, rows past the region read as zeros).
-//   warps 6-9  (the H2Share reuse step's variant) gather warps: a retrieval
-//              item's rows are borrowed positions, which these warps copy
-//              with 16-byte cp.async copies into the same swizzled ring, 32
-//              rows of each tile per warp; the CTAs split the step's rows
-//              with each gathered row weighing kGatherWeight contiguous rows
-//              (a row gather costs more than its share of a streamed tile).
+//   warps 6-21 (6-13 for G > 4; the H2Share reuse step's variant) gather
+//              warps: a retrieval item's rows are borrowed positions, which
+//              these warps copy with 16-byte cp.async copies into the same
+//              swizzled ring, 8 (16) rows of each tile per warp; the CTAs
+//              split the step's rows with each gathered row weighing 3/2
+//              contiguous rows (a row gather costs more than its share of a
+//              streamed tile). The MMA warp issues a gathered tile's P V
+//              right after its P, which frees the ring stage for the next
+//              gather one tile earlier.
 //   warp 5     TMEM owner and MMA issuer. Loads each item's Q into one of two
 //              swizzled buffers, writes the new token's K/V row over its
 //              (stale) cache row in the landed tile and appends it to the
@@ -54,7 +58,6 @@ constexpr int kBN = 128;                   // keys per tile
 constexpr int kN = 16;                     // N of both MMAs (query heads, padded)
 constexpr int kNS = 3;                     // ring stages
 constexpr int kThreads = 192;              // warps 0-5 (see the file comment)
-constexpr int kGatherWarps = 4;            // warps 6-9 of the H2Share reuse variant
 constexpr int kSoftmaxThreads = 128;
 constexpr uint32_t kTmemCols = 64;         // S[0] [0,16), S[1] [16,32), O [32,48)
 constexpr uint32_t kOcol = 32;
@@ -79,16 +82,25 @@ constexpr uint32_t IDESC_S = idesc_bf16(kBN, kN, false, false);
 constexpr uint32_t IDESC_PV = idesc_bf16(kD, kN, false, true);
 static_assert(SMEM <= 232448, "shared memory");
 static_assert(OFF_Q % 1024 == 0 && OFF_P % 1024 == 0, "operand alignment");
-static_assert((kThreads + 32 * kGatherWarps) * 8 <= kNS * kStage, "scan scratch");
 
-// GATHER: the H2Share reuse variant, whose four gather warps copy the borrowed
+// Gather warps of the H2Share reuse variant (warps 6 on). The cp.async
+// copies a warp keeps in flight are bounded per warp, so the gather rate
+// grows with the warps that issue them: sixteen for groups of up to four
+// heads (704 threads, 80 registers each), eight above, where the wider
+// group's softmax state needs more registers per thread.
+__host__ __device__ constexpr int gather_warps(int G, bool gather) { return gather ? (G <= 4 ? 16 : 8) : 0; }
+static_assert((kThreads + 32 * 16) * 8 <= kNS * kStage, "scan scratch");
+
+// GATHER: the H2Share reuse variant, whose gather warps copy the borrowed
 // rows of retrieval items (a.idx != nullptr); the producer warp then loads
 // only the contiguous (streaming) tiles.
 template <int G, bool GATHER>
-__global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1)
+__global__ void __launch_bounds__(kThreads + 32 * gather_warps(G, GATHER), 1)
     decode_tc_kernel(const __grid_constant__ DecodeArgs a) {
   static_assert(G >= 1 && G <= kN, "group size");
-  constexpr int NT = kThreads + (GATHER ? 32 * kGatherWarps : 0);
+  constexpr int GW = gather_warps(G, GATHER);
+  constexpr int RPW = GATHER ? kBN / GW : kBN;  // rows of each tile a gather warp copies
+  constexpr int NT = kThreads + 32 * GW;
   static_assert(2 * (dec::kGroup + 8) * G + 2 * G <= MS_FLOATS, "merge scratch");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
@@ -129,7 +141,7 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
     for (int s = 0; s < kNS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
-      mbar_init(&gfull[s], kGatherWarps);
+      mbar_init(&gfull[s], GATHER ? GW : 1);
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&s_full[x], 1);
@@ -210,22 +222,22 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
     __syncwarp();
   } else if (GATHER && warp >= 6) {
     // ------------------------------------------------------------ gatherers
-    // The reuse variant's four gather warps issue every tile of the CTA's
+    // The reuse variant's GW gather warps issue every tile of the CTA's
     // range, each of them waiting for every tile's stage to be free, in
     // order (an mbarrier parity wait is only sound within one phase of the
     // barrier, so no waiter may skip tiles). Contiguous (streaming) tiles:
     // lane 0 of warp 6 loads them with the TMA onto full[st]. Retrieval
-    // items: gather warp w copies rows 32 w .. 32 w + 31 of each 128-row tile
-    // of borrowed positions, one row per instruction (lanes 0-15 the 16
-    // chunks of its K row, lanes 16-31 those of its V row) with 16-byte
-    // cp.async copies into the swizzled layout the MMAs read, and the copies
-    // complete on gfull[st]; the new token's row (position t, not in the
-    // cache yet) comes from the step's input. Lane j holds the index of row
-    // 32 w + j, loaded two tiles ahead into one of two registers that
-    // alternate between tiles (a register copy of an in-flight load would
-    // wait for it). Row gathers through the TMA (tile::gather4 or bulk row
-    // copies) ran at about 15 GB/s per SM; cp.async copies scale with the
-    // issuing warps.
+    // items: gather warp w copies rows RPW w .. RPW w + RPW - 1 of each
+    // 128-row tile of borrowed positions, one row per instruction (lanes
+    // 0-15 the 16 chunks of its K row, lanes 16-31 those of its V row) with
+    // 16-byte cp.async copies into the swizzled layout the MMAs read, and the
+    // copies complete on gfull[st]; the new token's row (position t, not in
+    // the cache yet) comes from the step's input. Lane j < RPW holds the
+    // index of row RPW w + j, loaded two tiles ahead into one of two
+    // registers that alternate between tiles (a register copy of an
+    // in-flight load would wait for it). Row gathers through the TMA
+    // (tile::gather4 or bulk row copies) ran at about 15 GB/s per SM;
+    // cp.async copies scale with the issuing warps.
     const int gw = warp - 6;
     const int half = lane >> 4, ch = lane & 15;
     const uint32_t dst_lane = half * kTile + (ch >> 3) * kBox;
@@ -276,20 +288,21 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
           static_cast<const bf16*>(a.kv) + g.r_region(b, k) + (half ? (size_t)g.max_seq * kD : 0) + ch * 8;
       const bf16* src_new =
           static_cast<const bf16*>(half ? a.v_new : a.k_new) + ((size_t)b * g.Hkv + g.r_head[k]) * kD + ch * 8;
-      const int j0 = lo + 32 * gw + lane;
-      int ia = j0 < hi ? __ldg(rowlist + j0) : 0;
-      int ib = j0 + kBN < hi ? __ldg(rowlist + j0 + kBN) : 0;
+      const bool idx_lane = lane < RPW;
+      const int j0 = lo + RPW * gw + lane;
+      int ia = idx_lane && j0 < hi ? __ldg(rowlist + j0) : 0;
+      int ib = idx_lane && j0 + kBN < hi ? __ldg(rowlist + j0 + kBN) : 0;
       auto gather_tile = [&](int row0, int& buf) -> bool {
-        const int my_row = row0 + 32 * gw + lane < hi ? min(max(buf, 0), t) : -1;
-        const int jn = row0 + 2 * kBN + 32 * gw + lane;
-        buf = jn < hi ? __ldg(rowlist + jn) : 0;
+        const int my_row = idx_lane && row0 + RPW * gw + lane < hi ? min(max(buf, 0), t) : -1;
+        const int jn = row0 + 2 * kBN + RPW * gw + lane;
+        buf = idx_lane && jn < hi ? __ldg(rowlist + jn) : 0;
         const int st = it % kNS;
         if (!stage_free(st)) return false;
         uint8_t* tile = sKV + st * kStage + dst_lane;
 #pragma unroll 8
-        for (int j = 0; j < 32; ++j) {
+        for (int j = 0; j < RPW; ++j) {
           const int c = __shfl_sync(0xffffffffu, my_row, j);
-          const int r = 32 * gw + j;
+          const int r = RPW * gw + j;
           if (c >= 0)
             cp_async16(tile + r * 128 + ((swz ^ (uint32_t)(r & 7)) << 4),
                        c == t ? src_new : src_base + (size_t)c * kD);
@@ -483,6 +496,13 @@ __global__ void __launch_bounds__(kThreads + (GATHER ? 32 * kGatherWarps : 0), 1
         if (has_pend) issue_pv(pend);
         pend = Pend{it, st, item_k, row0 == lo};
         has_pend = true;
+        if (gathered) {
+          // a gathered tile's P V goes out as soon as its P is written:
+          // the next tile arrives late (random rows), and its stage is
+          // freed only by this P V
+          issue_pv(pend);
+          has_pend = false;
+        }
       }
       // Inside an item, P(j) V(j) waits behind S(j + 1) so that the softmax
       // of tile j + 1 can start meanwhile. At the item's end nothing can
@@ -702,7 +722,7 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
   // work on the stream itself (griddepcontrol.wait) after its prologue
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.n_ctas);
-  cfg.blockDim = dim3(kThreads + (GATHER ? 32 * kGatherWarps : 0));
+  cfg.blockDim = dim3(kThreads + 32 * gather_warps(G, GATHER));
   cfg.dynamicSmemBytes = SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -716,6 +736,12 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
 }  // namespace
 
 bool decode_uses_tc(int D, int G) { return D == kD && ((G >= 1 && G <= 8) || G == 16); }
+
+void reuse_tc_weights(int G, int* gather_w, int* ring_w) {
+  (void)G;
+  *gather_w = 3;
+  *ring_w = 2;
+}
 
 // One CTA per SM; small steps use fewer, at least 512 rows each.
 // At least 512 rows (four tiles) per CTA, so that small steps keep few

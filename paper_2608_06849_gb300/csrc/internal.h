@@ -90,9 +90,11 @@ struct DecodeArgs {
   const int32_t* idx = nullptr;
   int top_k = 0;
   int n_idx_groups = 0;
-  // Work units per gathered row when the CTAs split the step (a borrowed row
-  // costs several contiguous rows); 1 everywhere else.
+  // Work units per row when the CTAs split the reuse step: gather_w for a
+  // borrowed (gathered) row, ring_w for a contiguous one, so that a gathered
+  // row weighs gather_w / ring_w contiguous rows; both 1 in other steps.
   int gather_w = 1;
+  int ring_w = 1;
   uint8_t idx_map[kMaxKvHeads] = {};
 };
 
@@ -164,12 +166,13 @@ cudaError_t launch_h2_topk(float* ws, int max_seq, const int32_t* lens, int B, i
 int decode_ctas(long long total_rows, int num_sms, int D, int G);
 // The tcgen05 decode kernel serves (D, G) (else the CUDA-core kernel does).
 bool decode_uses_tc(int D, int G);
-// Work units of one gathered row in the reuse step's split on the tcgen05
-// kernel: a borrowed K and V row copied by the gather warps against a
-// contiguous row's share of a TMA tile stream (measured at 128K context,
-// top_k 2048: weights 2 / 3 / 4 / 5 gave 79.1 / 65.3 / 66.9 / 75.0 us at
-// B=16, 25.1 / 25.9 / 28.6 us at B=4).
-constexpr int kGatherWeight = 3;
+// Work units of a gathered row and of a contiguous row in the reuse step's
+// split on the tcgen05 kernel (a borrowed K and V row copied by the gather
+// warps against a contiguous row's share of a TMA tile stream), for group
+// size G. Measured at 128K context, top_k 2048, half the KV heads streaming:
+// gathered : contiguous = 3:2 / 5:3 / 2:1 / 3:1 gave 49 / 53 / 57 / - us at
+// g = 4, B = 16 (4:3 55 us), and 33.5 / - / 35 / 37 us at g = 7, B = 16.
+void reuse_tc_weights(int G, int* gather_w, int* ring_w);
 int decode_tc_ctas(long long total_rows, int num_sms);
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
