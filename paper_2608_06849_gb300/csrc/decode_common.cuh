@@ -55,15 +55,19 @@ __device__ __forceinline__ int item_weight(const DecodeArgs& a, int id) {
   if (a.idx == nullptr) return 1;
   return id % (a.geom.n_r + a.geom.n_s) < a.geom.n_r ? a.gather_w : a.ring_w;
 }
+// A non-empty item also carries a.item_cost units ahead of its first row:
+// the cost of switching to it, charged to the CTA whose range holds its
+// start.
 __device__ __forceinline__ long long item_units(const DecodeArgs& a, int id, const int* lens_s = nullptr) {
-  return (long long)item_rows(a, id, lens_s) * item_weight(a, id);
+  const int rows = item_rows(a, id, lens_s);
+  return rows > 0 ? (long long)rows * item_weight(a, id) + a.item_cost : 0;
 }
 
 // The rows of item `id` (at unit offset off) that the CTA with unit range
-// [start, end) owns: row r sits at unit off + r * w, so every row belongs to
-// exactly one CTA. lo >= hi when the CTA owns none.
+// [start, end) owns: row r sits at unit off + cost + r * w, so every row
+// belongs to exactly one CTA. lo >= hi when the CTA owns none.
 struct Span {
-  int rows, w, lo, hi;
+  int rows, w, cost, lo, hi;
   long long units;
 };
 __device__ __forceinline__ Span item_span(const DecodeArgs& a, int id, const int* lens_s, long long off,
@@ -71,8 +75,10 @@ __device__ __forceinline__ Span item_span(const DecodeArgs& a, int id, const int
   Span s;
   s.rows = item_rows(a, id, lens_s);
   s.w = item_weight(a, id);
-  s.units = (long long)s.rows * s.w;
-  const long long ulo = max(start, off) - off, uhi = min(end, off + s.units) - off;
+  s.cost = s.rows > 0 ? a.item_cost : 0;
+  s.units = (long long)s.rows * s.w + s.cost;
+  const long long base = off + s.cost;
+  const long long ulo = max(start, base) - base, uhi = min(end, base + (long long)s.rows * s.w) - base;
   s.lo = (int)((ulo + s.w - 1) / s.w);
   s.hi = uhi > ulo ? (int)((uhi + s.w - 1) / s.w) : s.lo;
   return s;

@@ -162,6 +162,7 @@ aoh_status noalloc_step(const aoh_config* cfg, const uint8_t* head_labels, void*
   a.gcounters = header + 64 + items;
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
   a.n_ctas = n_ctas;
+  if (decode_uses_tc(c.d_head, G)) a.item_cost = decode_tc_item_cost(total, n_ctas);
   a.self_clean = 1;
   a.status = header + kStatusWord;
   a.stall_cta = stall_cta;

@@ -95,6 +95,9 @@ struct DecodeArgs {
   // row weighs gather_w / ring_w contiguous rows; both 1 in other steps.
   int gather_w = 1;
   int ring_w = 1;
+  // Work units charged ahead of each non-empty item's first row (the cost of
+  // a CTA's switch to it), so the CTA that switches owns fewer rows.
+  int item_cost = 0;
   uint8_t idx_map[kMaxKvHeads] = {};
 };
 
@@ -173,6 +176,9 @@ bool decode_uses_tc(int D, int G);
 // gathered : contiguous = 3:2 / 5:3 / 2:1 / 3:1 gave 49 / 53 / 57 / - us at
 // g = 4, B = 16 (4:3 55 us), and 33.5 / - / 35 / 37 us at g = 7, B = 16.
 void reuse_tc_weights(int G, int* gather_w, int* ring_w);
+// DecodeArgs::item_cost for a plain or anchor step of the tcgen05 kernel
+// over total_rows rows on n_ctas CTAs (0 when each CTA's share is long).
+int decode_tc_item_cost(long long total_rows, int n_ctas);
 int decode_tc_ctas(long long total_rows, int num_sms);
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
