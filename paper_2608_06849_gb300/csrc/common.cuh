@@ -128,11 +128,15 @@ __device__ __forceinline__ void named_barrier_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
-// Release / acquire fence at GPU scope (lighter than the sequentially
-// consistent __threadfence). After a CTA barrier, one thread's fence orders
-// the whole CTA's earlier stores before its next relaxed atomic (release),
-// or that atomic before the CTA's later loads (acquire).
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+// Atomic add with acquire-release semantics at GPU scope. After a CTA
+// barrier, one thread's atomic publishes the whole CTA's earlier stores
+// (release) and orders the CTA's later loads, past the next barrier, after
+// it (acquire).
+__device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
 
 // Named barrier over `count` threads that also returns the AND of `pred`
 // over them (every thread of the barrier gets the same answer).

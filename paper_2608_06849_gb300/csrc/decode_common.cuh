@@ -295,9 +295,12 @@ template <int G, int D, int NT, bool WIDE>
 __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, int lst, int id,
                                            __nv_bfloat16* outp, float* scratch, volatile int* flag,
                                            float2* stats = nullptr) {
-  // the barrier orders every thread's partial stores before thread 0's fence
-  // and counter update (release); thread 0's fence after a last arrival
-  // orders the other parts' stores before the loads below (acquire)
+  // the barrier orders every thread's partial stores before thread 0's
+  // counter update, whose release half publishes them; its acquire half
+  // orders the other parts' stores before the loads below (the barrier
+  // that follows carries that to the other threads). One acq_rel atomic
+  // measured 2-4% faster per short step than a fence, a relaxed atomic and
+  // a second fence.
   named_barrier_sync(1, NT);
   const int np = lst - f + 1;
   const int gi = (p - f) / kGroup, p0 = f + gi * kGroup;
@@ -305,13 +308,9 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
   const int n_groups = (np + kGroup - 1) / kGroup;
   const int gslot = (p0 == f) ? 1 : 0;  // the item is p0's last item iff p0 == f
   if (threadIdx.x == 0) {
-    fence_acq_rel_gpu();
-    const uint32_t prev = atomicAdd(&a.gcounters[p0 * 2 + gslot], 1u);
+    const uint32_t prev = atom_add_acq_rel_gpu(&a.gcounters[p0 * 2 + gslot], 1u);
     const bool last = prev == (uint32_t)(gsz - 1);
-    if (last) {
-      fence_acq_rel_gpu();
-      a.gcounters[p0 * 2 + gslot] = 0u;
-    }
+    if (last) a.gcounters[p0 * 2 + gslot] = 0u;
     *flag = last;
   }
   named_barrier_sync(1, NT);
@@ -326,13 +325,9 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
   }
   merge_parts<G, D, NT, WIDE>(gsz, own, nullptr, partial_slot(a, p0, 2 + gslot, G, D), scratch);
   if (threadIdx.x == 0) {
-    fence_acq_rel_gpu();
-    const uint32_t prev = atomicAdd(&a.counters[id], 1u);
+    const uint32_t prev = atom_add_acq_rel_gpu(&a.counters[id], 1u);
     const bool last = prev == (uint32_t)(n_groups - 1);
-    if (last) {
-      fence_acq_rel_gpu();
-      a.counters[id] = 0u;
-    }
+    if (last) a.counters[id] = 0u;
     *flag = last;
   }
   named_barrier_sync(1, NT);
