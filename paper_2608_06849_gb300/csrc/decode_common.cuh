@@ -348,16 +348,15 @@ __device__ __forceinline__ void merge_item(const DecodeArgs& a, int p, int f, in
 // a self-cleaning launch zeroes them and the error word. The launch's flags
 // (timeout, capacity) are also ORed into the sticky status word when there
 // is one; nothing in a launch clears it. Only a launch that reads its flags
-// back (self-cleaning, or with a status word) needs the fences that make
-// every CTA's error-word updates visible to the last one; otherwise the
-// last CTA touches nothing another CTA wrote, and the next launch on the
-// stream starts after this grid has completed.
+// back (self-cleaning, or with a status word) needs its arrival to be an
+// acquire-release atomic, which makes every CTA's error-word updates
+// visible to the last one; otherwise the last CTA touches nothing another
+// CTA wrote. Either way the next launch on the stream starts after this
+// grid has completed, so nothing here needs a trailing fence.
 __device__ __forceinline__ void finish_launch(const DecodeArgs& a, const int* lens_s) {
   const bool readback = a.self_clean || a.status != nullptr;
-  if (readback) __threadfence();
-  const uint32_t prev = atomicAdd(a.done, 1u);
+  const uint32_t prev = readback ? atom_add_acq_rel_gpu(a.done, 1u) : atomicAdd(a.done, 1u);
   if (prev == gridDim.x - 1) {
-    if (readback) __threadfence();
     bool full = false;
     for (int i = 0; i < a.geom.B; ++i) {
       const int t = lens_s ? lens_s[i] : a.lens[i];
@@ -377,7 +376,6 @@ __device__ __forceinline__ void finish_launch(const DecodeArgs& a, const int* le
         *a.err = 0u;
       }
       if (!a.self_clean && full) atomicOr(a.err, kErrCapacity);
-      __threadfence();
     } else if (full) {
       atomicOr(a.err, kErrCapacity);
     }
