@@ -48,6 +48,11 @@ CASES = {
     "group5_d128": (2, 10, 2, 128, 260, 4, 50, [0, 1], [260, 131], 3),
     "group6_d128": (1, 12, 2, 128, 129, 2, 64, [1, 0], None, 3),
     "group16_d128": (1, 32, 2, 128, 400, 8, 100, [0, 1], None, 3),
+    # short decode steps charge each item's start in the CTA split: items of
+    # one to a few rows next to long ones, so CTA ranges cover several item
+    # starts and sometimes no row of an item
+    "tiny_items_with_item_charge": (12, 16, 4, 128, 3000, 4, 64, [0, 1, 0, 1],
+                                    [3000, 1, 2, 3, 700, 1, 1, 2500, 5, 1, 64, 129], 4),
 }
 
 
