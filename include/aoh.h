@@ -200,8 +200,9 @@ aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* 
  * Retrieval head i of sequence b attends to the first min(top_k, t + 1)
  * entries of its list; entries outside [0, t] are clamped into it (the
  * reads stay in bounds, the result is then unspecified). d_head 128 runs on
- * the tensor cores, the borrowed rows copied by four gather warps; d_head 64
- * on the CUDA-core kernel.
+ * the tensor cores, the borrowed rows copied by extra gather warps (sixteen
+ * for groups of up to four query heads, eight above); d_head 64 on the
+ * CUDA-core kernel.
  * Errors: INVALID, CAPACITY, UNSUPPORTED, CUDA.
  */
 aoh_status aoh_decode_step_reuse(const void* q, const void* k_new, const void* v_new, aoh_cache* cache,
