@@ -504,7 +504,12 @@ int decode_cc_ctas(long long total_rows, int num_sms) {
 
 size_t decode_partial_floats(int n_ctas, int G, int D) { return (size_t)n_ctas * 4 * dec::partial_stride(G, D); }
 
-cudaError_t launch_decode_cc(const DecodeArgs& a, cudaStream_t s) {
+cudaError_t launch_decode_cc(const DecodeArgs& args, cudaStream_t s) {
+  // this kernel walks its rows with unit weights and no item charge (its
+  // loops count rows, not work units), so the split must use the same
+  DecodeArgs a = args;
+  a.gather_w = a.ring_w = 1;
+  a.item_cost = 0;
   const int D = a.geom.D, G = a.geom.G;
   if (D == 128) {
     switch (G) {
