@@ -511,6 +511,7 @@ def run_native(args):
                     "cpu_baseline": pcpu},
         "chunked_prefill": {"chunks": n_chunks, "chunk_tokens": C, "ms": round(chunk_ms, 3),
                             "tflops": round(flops / (chunk_ms * 1e-3) / 1e12, 2),
+                            "frac": round(flops / (chunk_ms * 1e-3) / 1e12 / tf_peak, 4),
                             "note": "same 32K prefill as consecutive chunks; each chunk reads the cached prefix"},
         "chunk_eviction_prefill": {"chunk": C, "ms": round(evict_ms, 3), "flops": evict_flops,
                                    "tflops": round(evict_flops / (evict_ms * 1e-3) / 1e12, 2),
@@ -518,7 +519,7 @@ def run_native(args):
                                    "note": "the same chunks with aoh_config.chunk = C: streaming rows see the sinks, "
                                            "the W tokens before their chunk and the chunk (attended pairs counted "
                                            "under that rule)"},
-        "h2share": h2,
+        "h2share": dict(h2, reuse_frac_of_peak=round(h2["reuse_hbm_gbs"] / hbm_peak, 4)),
         "stack_256k": stack,
         "ragged_sweep": ragged,
         "e2e": {"value": round(e2e_us, 3), "unit": "us/step", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
