@@ -252,6 +252,10 @@ def _reuse_case(B, Hq, Hkv, D, T, S, W, labels, top_k, n_anchor, group_map, step
     (64, 16, 2, [1, 0], 33, 4, [3]),
     (128, 2, 2, [0, 1], 120, 2, [1]),            # groups of 1, gathered on the tensor cores
     (128, 32, 2, [0, 0], 300, 2, [1, 1]),        # groups of 16
+    (128, 4, 2, [0, 1], 180, 2, [1]),            # groups of 2 (sixteen gather warps)
+    (128, 6, 2, [1, 0], 260, 1, [0]),            # groups of 3
+    (128, 10, 2, [0, 0], 150, 2, [0, 1]),        # groups of 5 (eight gather warps)
+    (128, 16, 2, [0, 1], 400, 3, [2]),           # groups of 8
 ])
 def test_reuse_step_attends_to_borrowed_rows(D, Hq, Hkv, labels, top_k, n_anchor, gmap):
     _reuse_case(2, Hq, Hkv, D, 900, 4, 50, labels, top_k, n_anchor, gmap)
