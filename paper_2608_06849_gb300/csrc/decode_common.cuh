@@ -90,9 +90,11 @@ __device__ __forceinline__ int cta_of(long long x, long long total, int P) {
 }
 
 // Block-wide prefix sum of the items' rows (warp shuffles, then the warp
-// totals). On return (after the caller's next __syncthreads) sh64[0] = total
-// rows, sh64[1] = first row of the first item this CTA touches, sh32[0] =
-// that item. `wsum` is THREADS / 32 longs of scratch shared memory.
+// totals; up to 32 items, warp 0 alone, with no block barrier, which saves
+// ~0.4 us of a short step). On return (after the caller's next
+// __syncthreads) sh64[0] = total rows, sh64[1] = first row of the first item
+// this CTA touches, sh32[0] = that item. `wsum` is THREADS / 32 longs of
+// scratch shared memory.
 template <int THREADS>
 __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* wsum, long long* sh64, int* sh32,
                                                const int* lens_s = nullptr) {
@@ -101,6 +103,29 @@ __device__ __forceinline__ void find_cta_range(const DecodeArgs& a, long long* w
   const int n_items = g.B * (g.n_r + g.n_s);
   const int P = a.n_ctas, p = blockIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (n_items <= 32) {
+    // few items: warp 0 scans them alone (lane i holds item i)
+    if (warp == 0) {
+      const long long u = lane < n_items ? item_units(a, lane, lens_s) : 0;
+      long long inc = u;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      const long long total = __shfl_sync(0xffffffffu, inc, 31);
+      const long long start = (long long)p * total / P;
+      const unsigned past = __ballot_sync(0xffffffffu, lane < n_items && inc > start);
+      const int first = past ? __ffs(past) - 1 : n_items;
+      const long long excl = __shfl_sync(0xffffffffu, inc - u, first < 32 ? first : 31);
+      if (lane == 0) {
+        sh64[0] = total;
+        sh32[0] = first;
+        sh64[1] = first < n_items ? excl : total;
+      }
+    }
+    return;
+  }
   const int per = (n_items + THREADS - 1) / THREADS;
   const int i0 = min(n_items, (int)threadIdx.x * per), i1 = min(n_items, i0 + per);
   long long mine = 0;
