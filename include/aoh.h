@@ -363,11 +363,12 @@ aoh_status aoh_decode_step_noalloc_status(uint32_t* flags, void* stream);
 /*
  * Self-test of the allocation-free step's recovery from a bounded-wait
  * timeout (the paper has no counterpart): the same call and arguments as
- * aoh_decode_step_noalloc, except that in CTA 0 the softmax warps withhold
- * their first result, so the MMA warp's wait for it runs out (after about
- * 2 s) and that CTA stops once its copies and MMAs in flight have landed;
- * the other CTAs finish. The outputs of this call are unspecified, the new
- * token may be missing from the cache rows that CTA 0 would have appended,
+ * aoh_decode_step_noalloc, except that in the launch's last CTA (which
+ * always holds rows of the step) the softmax warps withhold their first
+ * result, so the MMA warp's wait for it runs out (after about 2 s) and that
+ * CTA stops once its copies and MMAs in flight have landed; the other CTAs
+ * finish. The outputs of this call are unspecified, the new token may be
+ * missing from the cache rows that the stalled CTA would have appended,
  * and the lengths advance as usual. The launch still leaves the static scratch clean, and
  * aoh_decode_step_noalloc_status() then reports AOH_ERR_TIMEOUT once.
  * Needs d_head 128 (UNSUPPORTED otherwise). Errors: as

@@ -474,7 +474,7 @@ aoh_status aoh_decode_step(const void* q, const void* k_new, const void* v_new, 
   if (st != AOH_OK) return st;
   const CacheGeom& g = cache->geom;
   a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
-  if (decode_uses_tc(g.D, g.G)) a.item_cost = decode_tc_item_cost(total, a.n_ctas);
+  if (decode_uses_tc(g.D, g.G)) a.item_cost = decode_tc_item_cost(total, a.n_ctas, cache->num_sms);
   cudaError_t e = launch_decode(a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");
   for (int b = 0; b < g.B; ++b) cache->lens[b] += 1;
@@ -498,7 +498,7 @@ aoh_status aoh_decode_step_anchor(const void* q, const void* k_new, const void* 
   }
   if (g.n_r > 0) h2_decode_outputs(cache->d_h2, g.B, g.n_r, g.G, g.max_seq, &a.scores, &a.score_stride, &a.score_stats);
   a.n_ctas = decode_ctas(total, cache->num_sms, g.D, g.G);
-  a.item_cost = decode_tc_item_cost(total, a.n_ctas);
+  a.item_cost = decode_tc_item_cost(total, a.n_ctas, cache->num_sms);
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e = launch_decode(a, s);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel launch");

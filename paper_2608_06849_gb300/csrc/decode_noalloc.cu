@@ -53,7 +53,8 @@ using namespace aoh;
 
 namespace {
 
-// The allocation-free step; stall_cta >= 0 runs the self-test.
+// The allocation-free step; stall_cta >= 0 runs the self-test (on the
+// launch's last CTA).
 aoh_status noalloc_step(const aoh_config* cfg, const uint8_t* head_labels, void* kv_buffer, int32_t* lens,
                         int32_t max_len, const void* q, const void* k_new, const void* v_new, void* out,
                         void* stream, int stall_cta) {
@@ -162,10 +163,12 @@ aoh_status noalloc_step(const aoh_config* cfg, const uint8_t* head_labels, void*
   a.gcounters = header + 64 + items;
   a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + kNoAllocHeaderBytes);
   a.n_ctas = n_ctas;
-  if (decode_uses_tc(c.d_head, G)) a.item_cost = decode_tc_item_cost(total, n_ctas);
+  if (decode_uses_tc(c.d_head, G)) a.item_cost = decode_tc_item_cost(total, n_ctas, num_sms);
   a.self_clean = 1;
   a.status = header + kStatusWord;
-  a.stall_cta = stall_cta;
+  // the self-test stalls the launch's last CTA: the step's last row is
+  // always its, whereas an item charge can leave the first CTAs without rows
+  a.stall_cta = stall_cta >= 0 ? n_ctas - 1 : -1;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)c.d_head));
   e = launch_decode(a, s);
   if (e != cudaSuccess) return set_err(AOH_ERR_CUDA, "aoh_decode_step_noalloc: kernel launch failed");

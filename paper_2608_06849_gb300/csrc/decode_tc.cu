@@ -65,18 +65,21 @@ constexpr float kRescaleThreshold = 8.0f;  // log2 units
 // Rows charged for a switch from one item to the next (DecodeArgs::
 // item_cost), in steps whose CTAs hold fewer than kItemCostMaxShare rows
 // each. A CTA that switches finishes its first item's epilogue and arrival
-// (a gpu-scope fence and an atomic) before the next item's softmax can go
-// on, so with an equal share it ends last and then also runs the second
-// item's merge. Measured with B=1, Qwen2.5-7B shape (2 of 4 KV heads
-// streaming), us per step, mean over six lengths T .. T + 331 (cost 0 /
-// 256 / 384 / 512 / 768 rows): 4K 16.9 / 16.9 / 16.2 / 15.4 / 14.9, 8K
-// 23.2 / 20.5 / 17.8 / 17.0 / 15.7, 16K 19.9 / 17.8 / 17.3 / 17.3 / 17.4,
-// 32K 21.7 / 18.1 / 18.0 / 17.8 / 17.8, 64K 24.7 / 23.8 / 22.7 / 22.9 /
-// 22.9, 128K 38.2 / - / 36.9 / 37.5 / 37.5; through the 28-layer stack per
-// token (CUDA graph; cost 0 / 384): 4K 467 / 480, 32K 675 / 582, 128K
-// 1092 / 1017. Llama-3-8B shape at B=16, 128K (29K rows per CTA): 628 us
-// with no cost, 629-630 with 256 rows.
+// before the next item's softmax can go on, so with an equal share it ends
+// last, and then also runs the second item's merge. Measured with B=1,
+// Qwen2.5-7B shape (2 of 4 KV heads streaming), us per step, mean over six
+// lengths T .. T + 331 (cost 0 / 256 / 384 / 512 / 768 rows): 4K 16.9 /
+// 16.9 / 16.2 / 15.4 / 14.9, 8K 23.2 / 20.5 / 17.8 / 17.0 / 15.7, 16K 19.9
+// / 17.8 / 17.3 / 17.3 / 17.4, 32K 21.7 / 18.1 / 18.0 / 17.8 / 17.8, 64K
+// 24.7 / 23.8 / 22.7 / 22.9 / 22.9, 128K 38.2 / - / 36.9 / 37.5 / 37.5;
+// through the 28-layer stack per token (CUDA graph; cost 384 / 512 / 768):
+// 4K 439 / 432 / 399, 32K 531 / 531 / 528, 128K 973 / 1037 / 1030.
+// Steps on fewer CTAs than SMs (4K, 8K: at least 512 rows per CTA, few
+// items) gain from the larger charge, which moves item starts onto CTA
+// boundaries; steps on every SM keep 384. Llama-3-8B shape at B=16, 128K
+// (29K rows per CTA): 628 us with no charge, 629-630 with 256 rows.
 constexpr int kItemCost = 384;
+constexpr int kItemCostFewCtas = 768;
 constexpr long long kItemCostMaxShare = 16384;
 constexpr int kBox = kBN * 64 * 2;         // one [128 rows][64] TMA box, 16 KB
 constexpr int kTile = 2 * kBox;            // a K or V tile (d = 128)
@@ -754,8 +757,9 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t s) {
 
 bool decode_uses_tc(int D, int G) { return D == kD && ((G >= 1 && G <= 8) || G == 16); }
 
-int decode_tc_item_cost(long long total_rows, int n_ctas) {
-  return total_rows < kItemCostMaxShare * n_ctas ? kItemCost : 0;
+int decode_tc_item_cost(long long total_rows, int n_ctas, int num_sms) {
+  if (total_rows >= kItemCostMaxShare * n_ctas) return 0;
+  return n_ctas < num_sms ? kItemCostFewCtas : kItemCost;
 }
 
 void reuse_tc_weights(int G, int* gather_w, int* ring_w) {

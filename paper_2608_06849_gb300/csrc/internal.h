@@ -177,8 +177,9 @@ bool decode_uses_tc(int D, int G);
 // g = 4, B = 16 (4:3 55 us), and 33.5 / - / 35 / 37 us at g = 7, B = 16.
 void reuse_tc_weights(int G, int* gather_w, int* ring_w);
 // DecodeArgs::item_cost for a plain or anchor step of the tcgen05 kernel
-// over total_rows rows on n_ctas CTAs (0 when each CTA's share is long).
-int decode_tc_item_cost(long long total_rows, int n_ctas);
+// over total_rows rows on n_ctas CTAs of a num_sms-SM GPU (0 when each
+// CTA's share is long).
+int decode_tc_item_cost(long long total_rows, int n_ctas, int num_sms);
 int decode_tc_ctas(long long total_rows, int num_sms);
 cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t s);
 // Floats of the partial buffer for `n_ctas` CTAs.
